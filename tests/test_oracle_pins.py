@@ -1,0 +1,340 @@
+"""Pins of the CPU oracle to things other than itself (no GPU needed).
+
+Each test ties one oracle function to the mathematics the paper fixes:
+brute force over the 0-1 program of Sec. III-B, closed forms of special cases,
+the optimality and ordering claims of Sec. IV-B3 and Sec. V-B, the one-
+dimensional form of Eq. 9, and the published test vector of SplitMix64.
+"""
+import math
+
+import numpy as np
+import pytest
+
+from conftest import read_golden
+from oracle import pyref
+from paper_2101_07968_gb300 import workloads as wl
+
+FWD, BWD = 0, 1
+
+
+def _prefix(v):
+    return np.concatenate([[0], np.cumsum(v)])
+
+
+def _cases(seed, n, lmax, kind):
+    rng = np.random.default_rng(seed)
+    for c in range(n):
+        L = int(rng.integers(1, lmax + 1))
+        gen = {"tie": wl.tie_heavy_instances, "uni": wl.random_instances,
+               "skew": wl.skewed_instances}[kind]
+        comp, xfer, dt = gen(seed * 1000 + c, 1, L)
+        yield comp[0], xfer[0], int(dt[0])
+
+
+# ------------------------------------------------------------------ brute force
+@pytest.mark.parametrize("kind", ["tie", "uni", "skew"])
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_dp_equals_brute_force(orc, kind, direction):
+    """Sec. IV-B3: the DP reaches the optimum of the 0-1 program (Sec. III-B);
+    the lowest-n final pick gives the fewest segments among optimal decisions;
+    the returned decision replays to the returned cost (f_m)."""
+    for comp, xfer, dt in _cases(11 + direction, 250, 11, kind):
+        v, d, s = orc.dp(direction, comp, xfer, dt)
+        bv, bs = orc.brute(direction, comp, xfer, dt)
+        assert v == bv, (comp, xfer, dt)
+        assert s == bs
+        assert 1 + int(d[1:len(comp)].sum()) == s
+        assert orc.replay(direction, comp, xfer, dt, d) == v
+
+
+def _literal_traceback_by_enumeration(orc, direction, comp, xfer, dt):
+    """The decision Algorithm 3/4 returns, derived without the recurrence:
+    opt(m, n) comes from enumerating every decision of the sub-problem; the
+    traceback starts at the fewest-segment optimum (L, s) and from (m, n) steps
+    to the LOWEST k for which some decision of (m, n) ending its previous
+    segment at k attains opt(m, n) -- the strict-improvement rule that keeps the
+    first minimising k, followed by Path."""
+    L = len(comp)
+    best, s, opt = orc.brute(direction, comp, xfer, dt, with_table=True)
+    d = [0] * (L + 1)
+    m, n = L, s
+    while n > 1:
+        found = None
+        for k in range(n - 1, m):
+            # best value of (m, n) whose previous segment ends at k: an optimal
+            # (k, n-1) prefix followed by one segment k+1..m
+            prev = opt[k][n - 1]
+            if direction == FWD:
+                P, FC = _prefix(xfer), _prefix(comp)
+                val = max(prev, n * dt + P[m]) + FC[m] - FC[k]
+            else:
+                SB, SG = _prefix(comp[::-1]), _prefix(xfer[::-1])
+                val = max(prev, SB[m]) + dt + SG[m] - SG[k]
+            if val == opt[m][n]:
+                found = k
+                break
+        assert found is not None
+        d[found] = 1
+        m, n = found, n - 1
+    return best, d, s
+
+
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_traceback_tie_break_by_enumeration(orc, direction):
+    """Pins the exact boundaries (not only the optimum) on tie-heavy inputs."""
+    for comp, xfer, dt in _cases(31 + direction, 300, 8, "tie"):
+        v, d, s = orc.dp(direction, comp, xfer, dt)
+        bv, bd, bs = _literal_traceback_by_enumeration(orc, direction, comp, xfer, dt)
+        assert (v, s) == (bv, bs)
+        assert list(d) == bd, (comp, xfer, dt)
+
+
+def test_subproblem_values_enumeration_consistency(orc):
+    """The enumeration's opt(m, n) satisfies Eq. 8's recurrence (forward) and
+    Eq. 9's (backward), i.e. the optimal-substructure claim of Sec. IV-B3."""
+    for direction in (FWD, BWD):
+        for comp, xfer, dt in _cases(41 + direction, 60, 7, "uni"):
+            L = len(comp)
+            _, _, opt = orc.brute(direction, comp, xfer, dt, with_table=True)
+            X = {(0, 0): 0}
+            for m in range(1, L + 1):
+                for n in range(1, m + 1):
+                    X[(m, n)] = int(opt[m][n])
+            for m in range(1, L + 1):
+                for n in range(1, m + 1):
+                    cands = []
+                    for k in range(0, m):
+                        if (k, n - 1) not in X:
+                            continue
+                        if direction == FWD:
+                            P, FC = _prefix(xfer), _prefix(comp)
+                            cands.append(max(X[(k, n - 1)], n * dt + P[m]) + FC[m] - FC[k])
+                        else:
+                            SB, SG = _prefix(comp[::-1]), _prefix(xfer[::-1])
+                            cands.append(max(X[(k, n - 1)], SB[m]) + dt + SG[m] - SG[k])
+                    assert min(cands) == X[(m, n)]
+
+
+# ------------------------------------------------------------ second transcription
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_python_transcription_agrees(orc, direction):
+    for kind in ("tie", "uni"):
+        for comp, xfer, dt in _cases(51 + direction, 150, 10, kind):
+            v, d, s = orc.dp(direction, comp, xfer, dt)
+            if direction == FWD:
+                pv, pd, ps = pyref.forward(list(xfer), list(comp), dt)
+            else:
+                pv, pd, ps = pyref.backward(list(comp), list(xfer), dt)
+            assert (v, s, list(d)) == (pv, ps, pd)
+
+
+# ----------------------------------------------------------------- closed forms
+def _flow_shop(a, b):
+    """Two-stage flow shop, fixed job order: max_j (sum_{i<=j} a_i + sum_{i>=j} b_i)."""
+    A, Bs = np.cumsum(a), np.cumsum(b[::-1])[::-1]
+    return int(max(A[j] + Bs[j] for j in range(len(a))))
+
+
+def test_replay_sequential_and_layer_by_layer_closed_forms(orc):
+    """f_m of the sequential strategy [0, L] and of layer-by-layer
+    [0, 1, ..., L] (Sec. III-B) in closed form."""
+    for comp, xfer, dt in _cases(61, 200, 20, "uni"):
+        L = len(comp)
+        seq = np.zeros(L + 1, np.uint8)
+        lbl = np.ones(L + 1, np.uint8)
+        lbl[0] = lbl[L] = 0
+        assert orc.replay(FWD, comp, xfer, dt, seq) == dt + xfer.sum() + comp.sum()
+        assert orc.replay(BWD, comp, xfer, dt, seq) == comp.sum() + dt + xfer.sum()
+        assert orc.replay(FWD, comp, xfer, dt, lbl) == _flow_shop(xfer + dt, comp)
+        # backward: layer L computes first; pushes in the same order
+        assert orc.replay(BWD, comp, xfer, dt, lbl) == _flow_shop(comp[::-1], xfer[::-1] + dt)
+
+
+def test_single_layer(orc):
+    for comp, xfer, dt in _cases(71, 50, 1, "uni"):
+        assert orc.dp(FWD, comp, xfer, dt)[0] == dt + xfer[0] + comp[0]
+        assert orc.dp(BWD, comp, xfer, dt)[0] == comp[0] + dt + xfer[0]
+        assert orc.dp(FWD, comp, xfer, dt)[2] == 1
+
+
+def test_zero_overhead_layer_by_layer_is_optimal(orc):
+    """dt = 0: splitting never delays an arrival, so layer-by-layer is optimal
+    and the optimum is the two-stage flow-shop makespan."""
+    for comp, xfer, _ in _cases(81, 200, 14, "uni"):
+        assert orc.dp(FWD, comp, xfer, 0)[0] == _flow_shop(xfer, comp)
+        assert orc.dp(BWD, comp, xfer, 0)[0] == _flow_shop(comp[::-1], xfer[::-1])
+
+
+def test_large_overhead_single_segment(orc):
+    """dt >= sum(comp) - comp of the last-processed layer: one transmission is
+    optimal, and the lowest-n pick returns the all-zero decision."""
+    for comp, xfer, _ in _cases(91, 200, 14, "uni"):
+        L = len(comp)
+        dtf = int(comp.sum() - comp[-1])
+        v, d, s = orc.dp(FWD, comp, xfer, dtf)
+        assert (v, s, int(d.sum())) == (dtf + xfer.sum() + comp.sum(), 1, 0)
+        dtb = int(comp.sum() - comp[L - 1])  # backward processes layer L first
+        v, d, s = orc.dp(BWD, comp, xfer, dtb)
+        assert (v, s, int(d.sum())) == (comp.sum() + dtb + xfer.sum(), 1, 0)
+
+
+# ------------------------------------------------------------------ invariants
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_not_worse_than_lbl_or_sequential_and_lower_bounds(orc, direction):
+    """Sec. V-B: DynaComm is never worse than LBL or Sequential."""
+    for kind in ("uni", "skew"):
+        for comp, xfer, dt in _cases(101 + direction, 150, 40, kind):
+            L = len(comp)
+            v, _, _ = orc.dp(direction, comp, xfer, dt)
+            seq = np.zeros(L + 1, np.uint8)
+            lbl = np.ones(L + 1, np.uint8)
+            lbl[0] = lbl[L] = 0
+            assert v <= orc.replay(direction, comp, xfer, dt, seq)
+            assert v <= orc.replay(direction, comp, xfer, dt, lbl)
+            if direction == FWD:
+                assert v >= dt + xfer[0] + comp.sum()
+                assert v >= dt + xfer.sum() + comp[-1]
+            else:
+                assert v >= comp.sum() + dt + xfer[0]
+                assert v >= comp[-1] + dt + xfer.sum()
+
+
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_monotone_in_every_cost_and_in_bandwidth(orc, direction):
+    rng = np.random.default_rng(7 + direction)
+    for comp, xfer, dt in _cases(111 + direction, 120, 25, "uni"):
+        L = len(comp)
+        v = orc.dp(direction, comp, xfer, dt)[0]
+        c2, x2 = comp.copy(), xfer.copy()
+        which = rng.integers(0, 3)
+        if which == 0:
+            c2[rng.integers(0, L)] += rng.integers(1, 500)
+        elif which == 1:
+            x2[rng.integers(0, L)] += rng.integers(1, 500)
+        assert orc.dp(direction, c2, x2, dt + (which == 2))[0] >= v
+        # lower bandwidth = every transfer cost scaled up
+        assert orc.dp(direction, comp, xfer * 3, dt)[0] >= v
+
+
+def test_backward_one_dimensional_form(orc):
+    """Eq. 9's cost ignores n, so min_n B[L][n] equals the 1-D recurrence."""
+    for kind in ("uni", "skew", "tie"):
+        for comp, xfer, dt in _cases(121, 80, 60, kind):
+            assert orc.dp(BWD, comp, xfer, dt)[0] == orc.dp_backward_1d(comp, xfer, dt)
+
+
+def test_infinite_bandwidth_limit(orc):
+    """pt = 0 (bandwidth -> infinity): the optimum is sum(fc) + the first
+    transfer (dt alone), and symmetric for the push."""
+    for comp, _, dt in _cases(131, 100, 30, "uni"):
+        z = np.zeros_like(comp)
+        assert orc.dp(FWD, comp, z, dt)[0] == dt + comp.sum()
+        assert orc.dp(BWD, comp, z, dt)[0] == comp.sum() + dt
+
+
+# ------------------------------------------------------------------- batches
+def test_batch_status_and_packing(orc):
+    comp, xfer, dt = wl.random_instances(5, 40, 37, 0, 10_000, 0, 1000)
+    comp[3, 5] = -1
+    dt[7] = -2
+    xfer[11, 0] = 1 << 52
+    out = orc.schedule_batch(FWD, comp, xfer, dt, nthreads=3)
+    assert out["status"][3] == 3 and out["makespan"][3] == -3 and out["nseg"][3] == 0
+    assert out["status"][7] == 3 and out["status"][11] == 4 and out["makespan"][11] == -4
+    assert not out["bits"][[3, 7, 11]].any()
+    for i in (0, 1, 2, 4, 39):
+        v, d, s = orc.dp(FWD, comp[i], xfer[i], dt[i])
+        assert out["makespan"][i] == v and out["nseg"][i] == s
+        assert np.array_equal(orc.bits_to_decision(out["bits"][i], 37), d)
+    rep = orc.replay_batch(FWD, comp, xfer, dt, out["bits"], nthreads=2)
+    ok = out["status"] == 0
+    assert np.array_equal(rep[ok], out["makespan"][ok])
+    assert rep[3] == -3 and rep[11] == -4
+
+
+# ------------------------------------------------------------------ generator
+def test_splitmix64_published_vector(orc):
+    for idx, value in read_golden("splitmix64_seed1234567.txt"):
+        assert orc.splitmix64(1234567, int(idx) - 1) == int(value)
+
+
+def test_standard_cnn_shapes():
+    for name, L, params, macs in read_golden("cnn_shapes.txt"):
+        c = wl.config(name)
+        assert c["L"] == int(L)
+        assert int(c["fixed_params"].sum()) == int(params)
+        assert int(c["fixed_flops"].sum()) == 2 * int(macs) * c["model_batch"]
+
+
+def test_uniform_int_distribution(orc):
+    rs = [orc.splitmix64(99, i) for i in range(20000)]
+    lo, hi = 10_000, 100_000
+    vals = np.array([orc.uniform_int(lo, hi, r) for r in rs])
+    assert vals.min() >= lo and vals.max() <= hi
+    sd = (hi - lo) / math.sqrt(12)
+    assert abs(vals.mean() - (lo + hi) / 2) < 5 * sd / math.sqrt(len(vals))
+    assert orc.uniform_int(lo, hi, 0) == lo and orc.uniform_int(lo, hi, 2**64 - 1) == hi
+    assert orc.uniform_int(5, 5, 12345) == 5
+
+
+def test_loguniform_distribution(orc):
+    rs = [orc.splitmix64(7, i) for i in range(20000)]
+    lo, hi = 1_000, 1_000_000
+    vals = np.array([orc.loguniform(lo, hi, r) for r in rs], dtype=np.float64)
+    assert vals.min() >= lo and vals.max() <= hi
+    logs = np.log(vals)
+    sd = (math.log(hi) - math.log(lo)) / math.sqrt(12)
+    assert abs(logs.mean() - (math.log(lo) + math.log(hi)) / 2) < 5 * sd / math.sqrt(len(vals))
+    # each decade holds a third of the mass
+    for a in (1e3, 1e4, 1e5):
+        frac = np.mean((vals >= a) & (vals < 10 * a))
+        assert abs(frac - 1 / 3) < 0.02
+    assert orc.loguniform(lo, hi, 0) == lo
+    assert orc.loguniform(lo, hi, 2**64 - 1) <= hi
+
+
+@pytest.mark.parametrize("name", ["tiny", "alexnet", "vgg16", "resnet50"])
+def test_generator_ceilings(orc, name):
+    """Each cost is the ceiling of work / speed: (c-1)*speed < work <= c*speed."""
+    cfg = wl.with_batch(wl.config(name), 64)
+    out = orc.profile_gen(cfg)
+    assert np.array_equal(out["pt"], out["gt"])
+    for i in range(0, 64, 7):
+        rate, bw, dt = orc.instance_draws(cfg, i)
+        assert cfg["rate_lo"] <= rate <= cfg["rate_hi"] and cfg["bw_lo"] <= bw <= cfg["bw_hi"]
+        assert out["dt"][i] == dt and cfg["dt_lo"] <= dt <= cfg["dt_hi"]
+        for l in range(cfg["L"]):
+            params = orc.layer_draw(cfg, i, 3, l)
+            flops = orc.layer_draw(cfg, i, 4, l)
+            if cfg["layer_mode"] == wl.LAYERS_FIXED:
+                assert params == cfg["fixed_params"][l] and flops == cfg["fixed_flops"][l]
+            else:
+                assert cfg["params_lo"] <= params <= cfg["params_hi"]
+                assert cfg["flops_lo"] <= flops <= cfg["flops_hi"]
+            for cost, work, speed in ((out["fc"][i, l], flops, rate),
+                                      (out["bc"][i, l], 2 * flops, rate),
+                                      (out["pt"][i, l], 32 * 1000 * params, bw)):
+                assert (cost - 1) * speed < work <= cost * speed
+
+
+def test_generator_is_counter_based(orc):
+    """An instance's profile depends on (seed, global index) only."""
+    cfg = wl.with_batch(wl.config("deepchain"), 9)
+    cfg["L"] = 40
+    full = orc.profile_gen(cfg)
+    part = orc.profile_gen(wl.with_batch(cfg, 3, inst0=5))
+    for k in ("fc", "pt", "bc", "gt", "dt"):
+        assert np.array_equal(full[k][5:8], part[k])
+    other = dict(cfg)
+    other["seed"] = 5
+    assert not np.array_equal(orc.profile_gen(other)["fc"], full["fc"])
+
+
+def test_generator_rejects_bad_config(orc):
+    cfg = wl.with_batch(wl.config("tiny"), 4)
+    for key, val in (("L", 0), ("L", 4097), ("rate_lo", 0), ("bw_hi", 2**31),
+                     ("bwd_flops_mult", 0), ("layer_mode", 9)):
+        bad = dict(cfg)
+        bad[key] = val
+        with pytest.raises(ValueError):
+            orc.profile_gen(bad)
