@@ -1,0 +1,421 @@
+"""Benchmark: batched DynaComm scheduling on GB300.
+
+One step = the whole scheduling path over one batch of synthetic instances:
+profile generation (dc_profile_gen), the forward DP (Eq. 8 / Algorithm 3), the
+backward DP (Eq. 9 / Algorithm 4) and the timeline replay f_m of both chosen
+decisions, with every input already resident in HBM. The end-to-end figure
+("e2e") runs the user-facing path instead: profiles in pinned host memory are
+copied in, scheduled and replayed, and the results are copied back, all inside
+the timed region.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload vgg16]
+    python bench.py --impl reference ...   # the CPU oracle on the host cores
+
+Prints one JSON line (rank 0). Under torchrun each rank solves its own batch of
+distinct instances (weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2101_07968_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "scheduling instances/s and DP cells/s on 1 GB300; % of int-ALU/HBM roofline"
+UNIT = "instances/s"
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_PATH = os.path.join(ROOT, "profiles", "dp_traffic.json")
+
+# Oracle sample sizes for the CPU baseline (instances per timed pass).
+CPU_SAMPLE = {"tiny": 4096, "alexnet": 1_000_000, "vgg16": 1_000_000, "resnet50": 65_536,
+              "deepchain": 16}
+
+
+def transitions(L: int) -> int:
+    """Finite (m, n, k) triples of one direction's DP: n = 1 has one candidate
+    per row; column n >= 2 has m - n + 1 candidates in row m."""
+    return L + (L + 1) * L * (L - 1) // 6
+
+
+def cells(L: int) -> int:
+    return L * (L + 1) // 2
+
+
+def dp_bytes(L: int) -> int:
+    """Algorithmic HBM bytes of one direction per instance: two cost rows and dt
+    in; makespan, decision words, nseg and status out."""
+    W = (L - 1 + 31) // 32
+    return 2 * L * 8 + 8 + 8 + 4 * W + 4 + 4
+
+
+# ------------------------------------------------------------------ helpers
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def load_json(path):
+    try:
+        with open(path) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return None
+
+
+def dp_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for name in ("dp_small.cu", "dp_group.cu", "common.cuh", "dynacomm_abi.cu"):
+        with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+# ------------------------------------------------------------- reference arm
+def oracle_pass(cfg, sample: int, nthreads: int):
+    """The oracle, as it stands, over the first `sample` instances of cfg:
+    generator, Algorithm 3, Algorithm 4 and f_m of both decisions."""
+    import oracle
+    c = wl.with_batch(cfg, sample, inst0=cfg.get("inst0", 0))
+    prof = oracle.profile_gen(c)
+    for d, (a, b) in ((0, ("fc", "pt")), (1, ("bc", "gt"))):
+        out = oracle.schedule_batch(d, prof[a], prof[b], prof["dt"], nthreads=nthreads)
+        oracle.replay_batch(d, prof[a], prof[b], prof["dt"], out["bits"], nthreads=nthreads)
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    cfg = wl.config(args.workload)
+    cores = os.cpu_count() or 1
+    sample = min(cfg["batch"], CPU_SAMPLE[args.workload])
+    for _ in range(args.warmup):
+        oracle_pass(cfg, sample, cores)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_pass(cfg, sample, cores)
+    dt = (time.perf_counter() - t0) / max(args.steps, 1)
+    value = sample / dt
+    desc = (f"first {sample} of {cfg['batch']} instances of {args.workload} per step: "
+            f"generator + Alg. 3 + Alg. 4 + f_m, {cores} threads")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": args.workload, "batch": cfg["batch"], "L": cfg["L"],
+                       "sample_per_step": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------- GPU arm
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2101_07968_gb300 import build as libbuild
+    from paper_2101_07968_gb300 import dynacomm as dc
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    libbuild.build()
+    dc.lib()
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    base = wl.config(args.workload)
+    B, L = base["batch"], base["L"]
+    cfg = wl.with_batch(base, B, inst0=rank * B)  # distinct instances per rank
+    W = dc.words(L)
+
+    prof = {k: torch.empty((B, L), dtype=torch.int64, device=dev) for k in ("fc", "pt", "bc", "gt")}
+    prof["dt"] = torch.empty(B, dtype=torch.int64, device=dev)
+    sched = dc.Scheduler(B, L, device=dev)
+    rep = {d: torch.empty(B, dtype=torch.int64, device=dev) for d in (0, 1)}
+    keep: list = []
+    ccfg = dc.make_cfg(cfg, keep)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record()
+        assert dc.dc_profile_gen(ccfg, prof["fc"], prof["pt"], prof["bc"], prof["gt"],
+                                 prof["dt"]) == 0
+        if ev is not None:
+            ev[1].record()
+        fo = sched.run(0, prof["fc"], prof["pt"], prof["dt"])
+        if ev is not None:
+            ev[2].record()
+        bo = sched.run(1, prof["bc"], prof["gt"], prof["dt"])
+        if ev is not None:
+            ev[3].record()
+        assert dc.dc_eval_timeline_batch(B, L, 0, prof["fc"], prof["pt"], prof["dt"],
+                                         fo["bits"], rep[0]) == 0
+        assert dc.dc_eval_timeline_batch(B, L, 1, prof["bc"], prof["gt"], prof["dt"],
+                                         bo["bits"], rep[1]) == 0
+        if ev is not None:
+            ev[4].record()
+
+    for _ in range(max(args.warmup, 0)):
+        step()
+    torch.cuda.synchronize()
+    # consistency of the path itself: replayed decisions reproduce the DP optimum
+    for d in (0, 1):
+        ok = torch.equal(rep[d], sched.out[d]["makespan"])
+        if not ok:
+            raise RuntimeError("timeline replay disagrees with the DP makespan")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index if rank == 0 else -1) if rank == 0 else _Null() as clk:
+        barrier()
+        torch.cuda.synchronize()
+        start.record()
+        for s in range(args.steps):
+            step(evs[s])
+        end.record()
+        torch.cuda.synchronize()
+        barrier()
+    ms = start.elapsed_time(end) / max(args.steps, 1)
+    seg = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])
+    gen_ms, fwd_ms, bwd_ms, eval_ms = seg.mean(axis=0)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # ---- ALU roof: the DP's transition op mix, register-only, all SMs
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    roof_threads, roof_blocks, roof_iters = 512, sms * 4, 20_000
+    sink = torch.empty(roof_blocks * roof_threads, dtype=torch.int32, device=dev)
+    roof = {}
+    for variant in (0, 1):
+        assert dc.dc_roof_int_probe(variant, roof_blocks, roof_threads, 400, sink) == 0
+        r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        r0.record()
+        assert dc.dc_roof_int_probe(variant, roof_blocks, roof_threads, roof_iters, sink) == 0
+        r1.record()
+        torch.cuda.synchronize()
+        roof[variant] = roof_blocks * roof_threads * roof_iters * 8 / (r0.elapsed_time(r1) * 1e-3)
+
+    # ---- end to end through the public API with host buffers
+    e2e = run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world)
+
+    # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        cores = os.cpu_count() or 1
+        sample = min(B, CPU_SAMPLE[args.workload])
+        t0 = time.perf_counter()
+        oracle_pass(base, sample, cores)
+        cpu_s = time.perf_counter() - t0
+        cpu = {"value": sample / cpu_s, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"first {sample} of {B} instances of {args.workload}: generator + "
+                         f"Alg. 3 + Alg. 4 + f_m, {cores} threads, {cpu_s:.1f} s"}
+
+    if rank != 0:
+        return 0
+    total = B * world
+    value = total / (ms * 1e-3)
+    trans = 2 * transitions(L) * B
+    dp_s = (fwd_ms + bwd_ms) * 1e-3
+    achieved = trans / dp_s / 1e9
+    peak = roof[0] / 1e9
+    traffic = None
+    tr = load_json(TRAFFIC_PATH)
+    if tr and tr.get("workload") == args.workload and tr.get("source_hash") == dp_source_hash():
+        traffic = tr.get("bytes_per_launch")
+    hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
+    dp_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
+    small = L <= 16
+    launches_per_step = 1 + 2 * (2 if small else 1) + 2
+    clocks = clk.summary() if rank == 0 else None
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": args.workload, "batch_per_gpu": B, "L": L,
+                   "global_batch": total,
+                   "l2": f"inputs larger than L2: {B * (4 * L + 1) * 8 / 1e6:.0f} MB of "
+                         "profiles written and re-read every step",
+                   "parallelism": f"independent instances, {world} GPU(s), no collective"},
+        "dp_cells_per_s": 2 * cells(L) * B * world / (ms * 1e-3),
+        "dp_transitions_per_s": trans * world / (ms * 1e-3),
+        "breakdown_ms": {"profile_gen": gen_ms, "dp_forward": fwd_ms, "dp_backward": bwd_ms,
+                         "eval_timeline_fwd_bwd": eval_ms},
+        "roofline": {"bound": "alu", "kernel": "dp_schedule (forward + backward)",
+                     "achieved": achieved, "peak": peak, "unit": "Gtransitions/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": "register-only probe of the same op mix (32-bit), "
+                                    f"{sms} SMs, measured in this run",
+                     "peak_u64": roof[1] / 1e9,
+                     "hbm": {"achieved_gbs": dp_gbs, "peak_gbs": hbm_peak,
+                             "frac": dp_gbs / hbm_peak,
+                             "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}},
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+class _Null:
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        return False
+
+    def summary(self):
+        return None
+
+
+def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
+    """Profiles in pinned host memory -> H2D -> forward + backward DP -> f_m of
+    both -> D2H of makespans, decisions and segment counts, every step."""
+    host_in = {k: v.cpu().pin_memory() for k, v in prof.items()}
+    dev_in = {k: torch.empty_like(v) for k, v in prof.items()}
+    rep = {d: torch.empty(B, dtype=torch.int64, device=dev) for d in (0, 1)}
+    host_out = {}
+    for d in (0, 1):
+        for k in ("makespan", "bits", "nseg"):
+            host_out[(d, k)] = torch.empty_like(sched.out[d][k], device="cpu").pin_memory()
+        host_out[(d, "replay")] = torch.empty(B, dtype=torch.int64).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in host_in.values())
+    d2h = sum(v.numel() * v.element_size() for v in host_out.values())
+
+    def e2e_step():
+        for k in host_in:
+            dev_in[k].copy_(host_in[k], non_blocking=True)
+        fo = sched.run(0, dev_in["fc"], dev_in["pt"], dev_in["dt"])
+        bo = sched.run(1, dev_in["bc"], dev_in["gt"], dev_in["dt"])
+        assert dc.dc_eval_timeline_batch(B, L, 0, dev_in["fc"], dev_in["pt"], dev_in["dt"],
+                                         fo["bits"], rep[0]) == 0
+        assert dc.dc_eval_timeline_batch(B, L, 1, dev_in["bc"], dev_in["gt"], dev_in["dt"],
+                                         bo["bits"], rep[1]) == 0
+        for d, o in ((0, fo), (1, bo)):
+            for k in ("makespan", "bits", "nseg"):
+                host_out[(d, k)].copy_(o[k], non_blocking=True)
+            host_out[(d, "replay")].copy_(rep[d], non_blocking=True)
+
+    for _ in range(max(args.warmup, 1)):
+        e2e_step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, 5))
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        e2e_step()
+    t1.record()
+    torch.cuda.synchronize()
+    barrier()
+    ms = t0.elapsed_time(t1) / steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": B * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps,
+            "path": "pinned host profiles -> dc_schedule_forward/backward_batch -> "
+                    "dc_eval_timeline_batch -> pinned host results"}
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", choices=list(wl.CONFIG_NAMES), default="vgg16")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    args = p.parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

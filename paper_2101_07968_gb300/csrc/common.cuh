@@ -1,0 +1,98 @@
+// Shared device/host helpers of the GB300 DynaComm library (GPU side only).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "dynacomm.h"
+
+namespace dc {
+
+constexpr int kSmallLMax = 16;       // thread-per-instance kernel covers 1 <= L <= 16
+constexpr int kSmemTableLMax = 64;   // group kernel keeps its DP table on chip up to here
+constexpr int64_t kRangeLimit = int64_t(1) << 52;
+constexpr uint64_t kNarrowLimit = 0xFFFFFFFEull;  // bound that lets a DP run in 32 bits
+
+// Triangle of DP cells (m, n), 1 <= n <= m <= L, stored column by column:
+// column n holds rows n..L contiguously.
+__host__ __device__ inline int64_t tri_cells(int L) { return int64_t(L) * (L + 1) / 2; }
+__host__ __device__ inline int64_t tri_col(int L, int n)
+{
+    return int64_t(n - 1) * L - int64_t(n - 1) * (n - 2) / 2;
+}
+__host__ __device__ inline int64_t tri_index(int L, int m, int n) { return tri_col(L, n) + (m - n); }
+
+__host__ __device__ inline int words_for(int L) { return (L - 1 + 31) / 32; }
+
+// Group-kernel table slots (L > kSmemTableLMax): enough CTAs to fill the GPU
+// several times over, capped so one launch's tables stay within ~4 GiB.
+inline int64_t table_slots(int L)
+{
+    const int64_t per = tri_cells(L) * 8;
+    int64_t s = (int64_t(4) << 30) / per;
+    if (s > 1024) s = 1024;
+    if (s < 152) s = 152;
+    return s;
+}
+
+struct Workspace {
+    // Layout: [0, 256) header (wide-list counter), [256, 256 + 4*batch) wide list
+    // (only when L <= kSmallLMax), then 256-aligned per-slot DP tables (L > 64).
+    static size_t list_bytes(int64_t batch, int L)
+    {
+        return L <= kSmallLMax ? size_t(batch) * 4 : 0;
+    }
+    static size_t table_offset(int64_t batch, int L)
+    {
+        return (256 + list_bytes(batch, L) + 255) / 256 * 256;
+    }
+    static size_t slots(int64_t batch, int L)
+    {
+        if (L <= kSmemTableLMax) return 0;
+        int64_t s = table_slots(L);
+        return size_t(batch < s ? batch : s);
+    }
+    static size_t bytes(int64_t batch, int L)
+    {
+        return table_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
+    }
+};
+
+// L*dt + sum(comp) + sum(xfer) >= 2^52, for inputs already known to be
+// non-negative and below 2^52 each (so each sum of <= 4096 terms fits 64 bits).
+__host__ __device__ inline bool exceeds_range(int L, int64_t dt, uint64_t sc, uint64_t sx)
+{
+    const uint64_t lim = uint64_t(kRangeLimit);
+    if (sc >= lim || sx >= lim) return true;
+    const uint64_t tl = uint64_t(L) * uint64_t(dt);
+    return tl >= lim || sc + sx + tl >= lim;
+}
+
+template <typename T>
+__device__ __forceinline__ T dmax(T a, T b) { return a > b ? a : b; }
+template <typename T>
+__device__ __forceinline__ T dmin(T a, T b) { return a < b ? a : b; }
+
+// Kernel launchers implemented in the .cu files.
+cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *comp,
+                            const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                            uint32_t *bits, int32_t *nseg, int32_t *status, void *workspace,
+                            cudaStream_t stream);
+cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp,
+                         const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                         uint32_t *bits, int32_t *nseg, int32_t *status,
+                         uint32_t *wide_count, uint32_t *wide_list, cudaStream_t stream);
+cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp,
+                         const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                         uint32_t *bits, int32_t *nseg, int32_t *status,
+                         const uint32_t *list_count, const uint32_t *list, void *tables,
+                         int64_t grid, cudaStream_t stream);
+cudaError_t launch_eval(bool forward, int64_t batch, int L, const int64_t *comp,
+                        const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
+                        int64_t *makespan, cudaStream_t stream);
+cudaError_t launch_roof(int variant, int blocks, int threads, int64_t iters, uint32_t *sink,
+                        cudaStream_t stream);
+
+}  // namespace dc

@@ -1,0 +1,308 @@
+// CTA-per-instance DynaComm DP for any 1 <= L <= 4096 (Eq. 8 / Algorithm 3 and
+// Eq. 9 / Algorithm 4), in 32-bit or 64-bit arithmetic per instance.
+//
+// Used for L > 16, and for the L <= 16 instances whose values need 64 bits
+// (the thread-per-instance kernel puts those on a work list).
+//
+// Same processing-order template as the small kernel:
+//   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
+// Column n is filled in parallel (one row m per thread, strided), columns run in
+// sequence with a CTA barrier between them; two column buffers live in shared
+// memory and every finished cell is also written to the instance's DP table
+// (shared memory for L <= 64, otherwise a per-CTA slot of the caller's
+// workspace). After the fill, warp 0 picks the lowest n minimising X[L][n] and
+// walks the traceback, finding each Path[m][n] (the lowest k whose candidate
+// equals the cell) with one ballot per 32 candidates.
+#include "common.cuh"
+
+namespace dc {
+namespace {
+
+struct GroupArgs {
+    int64_t batch;
+    int L;
+    const int64_t *comp, *xfer, *dt;
+    int64_t *makespan;
+    uint32_t *bits;
+    int32_t *nseg, *status;
+    const uint32_t *list_count, *list;
+    unsigned char *tables;  // nullptr: DP table in shared memory
+};
+
+// Shared-memory layout: four (L+1)-entry arrays sized for 64-bit values
+// (S, R, two column buffers), the decision words, a 256-byte scan scratch, and
+// the DP table when it stays on chip.
+__host__ __device__ inline size_t group_arrays_bytes(int L) { return size_t(4) * (L + 1) * 8; }
+__host__ __device__ inline size_t group_bits_bytes(int L)
+{
+    return (size_t(words_for(L) + 1) * 4 + 15) / 16 * 16;
+}
+constexpr size_t kScratchBytes = 256;
+__host__ __device__ inline size_t group_table_offset(int L)
+{
+    return group_arrays_bytes(L) + group_bits_bytes(L) + kScratchBytes;
+}
+inline size_t group_smem_bytes(int L, bool table_in_smem)
+{
+    return group_table_offset(L) + (table_in_smem ? size_t(tri_cells(L)) * 8 : 0);
+}
+
+// Inclusive prefix of v[1..L] in place (v[0] = 0), CTA-wide; each thread owns
+// a contiguous chunk, chunk totals are scanned by warp 0.
+__device__ void block_prefix_u64(uint64_t *v, int L, uint64_t *scratch /* >= 16 entries */)
+{
+    const int nt = blockDim.x, t = threadIdx.x;
+    const int chunk = (L + nt - 1) / nt;
+    const int lo = 1 + t * chunk, hi = min(L, lo + chunk - 1);
+    uint64_t acc = 0;
+    for (int j = lo; j <= hi; ++j) {
+        acc += v[j];
+        v[j] = acc;
+    }
+    // exclusive scan of per-thread totals: warp-level, then across warps
+    const int lane = t & 31, warp = t >> 5, nw = (nt + 31) >> 5;
+    uint64_t x = acc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint64_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) scratch[warp] = x;
+    __syncthreads();
+    if (t == 0) {
+        uint64_t run = 0;
+        for (int w = 0; w < nw; ++w) {
+            const uint64_t tot = scratch[w];
+            scratch[w] = run;
+            run += tot;
+        }
+    }
+    __syncthreads();
+    const uint64_t off = scratch[warp] + x - acc;
+    for (int j = lo; j <= hi; ++j) v[j] += off;
+    __syncthreads();
+}
+
+template <typename T, bool FWD>
+__device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, const uint64_t *P64c,
+                      const uint64_t *P64x, unsigned char *arrays, uint32_t *bitsw,
+                      T *table)
+{
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x;
+    T *S = reinterpret_cast<T *>(arrays);
+    T *Rb = S + (L + 1);
+    T *colA = Rb + (L + 1);
+    T *colB = colA + (L + 1);
+    // P64c / P64x sit in the 64-bit column-buffer bytes, past the typed S and R
+    // arrays for either T; the typed columns overwrite them only after this copy.
+    for (int m = t; m <= L; m += nt) {
+        S[m] = T(FWD ? P64c[m] : P64x[m]);
+        Rb[m] = T(FWD ? P64x[m] : P64c[m]);
+    }
+    __syncthreads();
+
+    const T dtv = T(dti);
+    const T c = FWD ? T(0) : dtv;
+    // column 1
+    for (int m = 1 + t; m <= L; m += nt) {
+        const T R = FWD ? T(dtv + Rb[m]) : Rb[m];
+        const T v = T(R + S[m] + c);
+        colA[m] = v;
+        table[tri_index(L, m, 1)] = v;
+    }
+    __syncthreads();
+    T *prev = colA, *cur = colB;
+    for (int n = 2; n <= L; ++n) {
+        const T ndt = T(T(n) * dtv);
+        const int64_t cbase = tri_col(L, n) - n;
+        for (int m = n + t; m <= L; m += nt) {
+            const T R = FWD ? T(ndt + Rb[m]) : Rb[m];
+            T best = T(dmax(prev[n - 1], R) - S[n - 1]);
+            int k = n;
+            for (; k + 3 < m; k += 4) {
+                const T c0 = T(dmax(prev[k], R) - S[k]);
+                const T c1 = T(dmax(prev[k + 1], R) - S[k + 1]);
+                const T c2 = T(dmax(prev[k + 2], R) - S[k + 2]);
+                const T c3 = T(dmax(prev[k + 3], R) - S[k + 3]);
+                best = dmin(best, dmin(dmin(c0, c1), dmin(c2, c3)));
+            }
+            for (; k < m; ++k) best = dmin(best, T(dmax(prev[k], R) - S[k]));
+            const T v = T(best + S[m] + c);
+            cur[m] = v;
+            table[cbase + m] = v;
+        }
+        __syncthreads();
+        T *tmp = prev;
+        prev = cur;
+        cur = tmp;
+    }
+
+    // final pick and traceback by warp 0
+    if (t < 32) {
+        const int lane = t;
+        T bv = T(~T(0));
+        int bn = 0x7fffffff;
+        for (int n = 1 + lane; n <= L; n += 32) {
+            const T v = table[tri_index(L, L, n)];
+            if (v < bv) {  // n increases: strict keeps the lowest n in this lane
+                bv = v;
+                bn = n;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const T ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int on = __shfl_xor_sync(0xffffffffu, bn, o);
+            if (ov < bv || (ov == bv && on < bn)) {
+                bv = ov;
+                bn = on;
+            }
+        }
+        const int s = bn;
+        int err = 0;
+        int m = L, n = s;
+        while (n > 1) {
+            const T R = FWD ? T(T(n) * dtv + Rb[m]) : Rb[m];
+            const T target = T(table[tri_index(L, m, n)] - S[m] - c);
+            const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
+            int found = -1;
+            for (int k0 = n - 1; k0 < m; k0 += 32) {
+                const int k = k0 + lane;
+                bool match = false;
+                if (k < m) match = T(dmax(table[pbase + k], R) - S[k]) == target;
+                const unsigned bal = __ballot_sync(0xffffffffu, match);
+                if (bal) {
+                    found = k0 + __ffs(bal) - 1;
+                    break;
+                }
+            }
+            if (found < 0) {
+                err = 1;
+                break;
+            }
+            if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
+            __syncwarp();
+            m = found;
+            n -= 1;
+        }
+        if (lane == 0) {
+            a.makespan[i] = int64_t(bv);
+            if (a.nseg) a.nseg[i] = s;
+            if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+        }
+    }
+    __syncthreads();
+}
+
+template <bool FWD>
+__global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x;
+    const int W = words_for(L);
+    unsigned char *arrays = smem;
+    uint32_t *bitsw = reinterpret_cast<uint32_t *>(smem + group_arrays_bytes(L));
+    uint64_t *scratch =
+        reinterpret_cast<uint64_t *>(smem + group_arrays_bytes(L) + group_bits_bytes(L));
+    unsigned char *smem_table = smem + group_table_offset(L);
+    unsigned char *slot =
+        a.tables ? a.tables + size_t(blockIdx.x) * size_t(tri_cells(L)) * 8 : smem_table;
+    // 64-bit prefix arrays live in the column buffers until the typed copy.
+    uint64_t *P64c = reinterpret_cast<uint64_t *>(arrays) + 2 * (L + 1);
+    uint64_t *P64x = P64c + (L + 1);
+
+    const int64_t count = a.list_count ? int64_t(*a.list_count) : a.batch;
+    for (int64_t j = blockIdx.x; j < count; j += gridDim.x) {
+        const int64_t i = a.list ? int64_t(a.list[j]) : j;
+        const int64_t *crow = a.comp + i * L;
+        const int64_t *xrow = a.xfer + i * L;
+        const int64_t dti = a.dt[i];
+        int bad_neg = dti < 0, bad_big = (dti >> 52) != 0;
+        for (int r = 1 + t; r <= L; r += nt) {
+            const int col = FWD ? r - 1 : L - r;
+            const int64_t cv = __ldg(crow + col), xv = __ldg(xrow + col);
+            bad_neg |= (cv < 0) | (xv < 0);
+            bad_big |= ((cv | xv) >> 52) != 0;
+            P64c[r] = uint64_t(cv);
+            P64x[r] = uint64_t(xv);
+        }
+        for (int w = t; w < W; w += nt) bitsw[w] = 0u;
+        if (t == 0) {
+            P64c[0] = 0;
+            P64x[0] = 0;
+        }
+        const int any_neg = __syncthreads_or(bad_neg);
+        const int any_big = __syncthreads_or(bad_big);
+        int st = DC_OK;
+        bool narrow = false;
+        if (any_neg) {
+            st = DC_ERR_NEGATIVE;
+        } else if (any_big) {
+            st = DC_ERR_RANGE;
+        } else {
+            block_prefix_u64(P64c, L, scratch);
+            block_prefix_u64(P64x, L, scratch);
+            const uint64_t tc = P64c[L], tx = P64x[L];
+            if (exceeds_range(L, dti, tc, tx))
+                st = DC_ERR_RANGE;
+            else
+                narrow = tc + tx + uint64_t(L) * uint64_t(dti) <= kNarrowLimit;
+        }
+        if (st != DC_OK) {
+            if (t == 0) {
+                a.makespan[i] = -int64_t(st);
+                if (a.nseg) a.nseg[i] = 0;
+                if (a.status) a.status[i] = st;
+            }
+            for (int w = t; w < W; w += nt) a.bits[i * W + w] = 0u;
+            __syncthreads();
+            continue;
+        }
+        if (narrow)
+            solve<uint32_t, FWD>(a, i, dti, P64c, P64x, arrays, bitsw,
+                                 reinterpret_cast<uint32_t *>(slot));
+        else
+            solve<uint64_t, FWD>(a, i, dti, P64c, P64x, arrays, bitsw,
+                                 reinterpret_cast<uint64_t *>(slot));
+        for (int w = t; w < W; w += nt) a.bits[i * W + w] = bitsw[w];
+        __syncthreads();
+    }
+}
+
+int group_threads(int L)
+{
+    if (L <= 64) return 64;
+    if (L <= 256) return 128;
+    if (L <= 1024) return 256;
+    return 512;
+}
+
+}  // namespace
+
+cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp,
+                         const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                         uint32_t *bits, int32_t *nseg, int32_t *status,
+                         const uint32_t *list_count, const uint32_t *list, void *tables,
+                         int64_t grid, cudaStream_t stream)
+{
+    if (grid <= 0) return cudaSuccess;
+    GroupArgs a{batch, L, comp, xfer, dt, makespan, bits, nseg, status, list_count, list,
+                static_cast<unsigned char *>(tables)};
+    const size_t smem = group_smem_bytes(L, tables == nullptr);
+    const int nt = group_threads(L);
+    cudaError_t e;
+    if (forward) {
+        e = cudaFuncSetAttribute(group_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(smem));
+        if (e != cudaSuccess) return e;
+        group_kernel<true><<<unsigned(grid), nt, smem, stream>>>(a);
+    } else {
+        e = cudaFuncSetAttribute(group_kernel<false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (e != cudaSuccess) return e;
+        group_kernel<false><<<unsigned(grid), nt, smem, stream>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace dc

@@ -1,0 +1,144 @@
+// C ABI entry points (declared in include/dynacomm.h): host-side argument
+// checks, then kernel launches on the caller's stream. No allocation, no
+// synchronisation, no state kept between calls.
+#include "common.cuh"
+
+namespace dc {
+
+dc_status check_profile_cfg(const dc_profile_cfg *c);
+cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_t *bc,
+                       int64_t *gt, int64_t *dt, cudaStream_t stream);
+
+// Forward and backward solves share one path after the layers are put in
+// processing order (done inside the kernels).
+cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *comp,
+                            const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                            uint32_t *bits, int32_t *nseg, int32_t *status, void *workspace,
+                            cudaStream_t stream)
+{
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    if (L <= kSmallLMax) {
+        uint32_t *count = reinterpret_cast<uint32_t *>(ws);
+        uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
+        cudaError_t e = cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
+        if (e != cudaSuccess) return e;
+        e = launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, count,
+                         list, stream);
+        if (e != cudaSuccess) return e;
+        // 64-bit leftovers: a persistent grid that reads the list length on the device
+        const int64_t grid = batch < 1216 ? batch : 1216;
+        return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                            count, list, nullptr, grid, stream);
+    }
+    if (L <= kSmemTableLMax) {
+        const int64_t grid = batch < 152 * 32 ? batch : 152 * 32;
+        return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                            nullptr, nullptr, nullptr, grid, stream);
+    }
+    const int64_t slots = int64_t(Workspace::slots(batch, L));
+    return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                        nullptr, nullptr, ws + Workspace::table_offset(batch, L), slots,
+                        stream);
+}
+
+namespace {
+
+dc_status schedule(bool forward, int64_t batch, int32_t L, const int64_t *comp,
+                   const int64_t *xfer, const int64_t *dt, int64_t *makespan, uint32_t *bits,
+                   int32_t *nseg, int32_t *status, void *workspace, size_t workspace_bytes,
+                   cudaStream_t stream)
+{
+    if (batch < 0 || L < 1 || L > DC_L_MAX || batch > int64_t(0xffffffffll))
+        return DC_ERR_BAD_SHAPE;
+    if (batch == 0) return DC_OK;
+    if (!comp || !xfer || !dt || !makespan || (!bits && words_for(L) > 0)) return DC_ERR_NULL;
+    if (!workspace || workspace_bytes < Workspace::bytes(batch, L)) return DC_ERR_WORKSPACE;
+    const cudaError_t e = launch_schedule(forward, batch, L, comp, xfer, dt, makespan, bits,
+                                          nseg, status, workspace, stream);
+    return e == cudaSuccess ? DC_OK : DC_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace dc
+
+extern "C" {
+
+dc_status dc_profile_gen(const dc_profile_cfg *cfg, int64_t *fc, int64_t *pt, int64_t *bc,
+                         int64_t *gt, int64_t *dt, cudaStream_t stream)
+{
+    if (!cfg) return DC_ERR_NULL;
+    const dc_status st = dc::check_profile_cfg(cfg);
+    if (st != DC_OK) return st;
+    if (cfg->batch == 0) return DC_OK;
+    if (!fc || !pt || !bc || !gt || !dt) return DC_ERR_NULL;
+    return dc::launch_gen(cfg, fc, pt, bc, gt, dt, stream) == cudaSuccess ? DC_OK : DC_ERR_CUDA;
+}
+
+size_t dc_schedule_workspace_bytes(int64_t batch, int32_t L)
+{
+    if (batch < 0 || L < 1 || L > DC_L_MAX) return 0;
+    return dc::Workspace::bytes(batch, L);
+}
+
+dc_status dc_schedule_forward_batch(int64_t batch, int32_t L, const int64_t *fc,
+                                    const int64_t *pt, const int64_t *dt, int64_t *makespan,
+                                    uint32_t *bits, int32_t *nseg, int32_t *status,
+                                    void *workspace, size_t workspace_bytes, cudaStream_t stream)
+{
+    return dc::schedule(true, batch, L, fc, pt, dt, makespan, bits, nseg, status, workspace,
+                        workspace_bytes, stream);
+}
+
+dc_status dc_schedule_backward_batch(int64_t batch, int32_t L, const int64_t *bc,
+                                     const int64_t *gt, const int64_t *dt, int64_t *makespan,
+                                     uint32_t *bits, int32_t *nseg, int32_t *status,
+                                     void *workspace, size_t workspace_bytes,
+                                     cudaStream_t stream)
+{
+    return dc::schedule(false, batch, L, bc, gt, dt, makespan, bits, nseg, status, workspace,
+                        workspace_bytes, stream);
+}
+
+dc_status dc_eval_timeline_batch(int64_t batch, int32_t L, int32_t dir, const int64_t *comp,
+                                 const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
+                                 int64_t *makespan, cudaStream_t stream)
+{
+    if (batch < 0 || L < 1 || L > DC_L_MAX || (dir != 0 && dir != 1)) return DC_ERR_BAD_SHAPE;
+    if (batch == 0) return DC_OK;
+    if (!comp || !xfer || !dt || !makespan || (!bits && dc::words_for(L) > 0))
+        return DC_ERR_NULL;
+    return dc::launch_eval(dir == 0, batch, L, comp, xfer, dt, bits, makespan, stream) ==
+                   cudaSuccess
+               ? DC_OK
+               : DC_ERR_CUDA;
+}
+
+const char *dc_status_string(dc_status s)
+{
+    switch (s) {
+        case DC_OK: return "ok";
+        case DC_ERR_NULL: return "a required pointer is NULL";
+        case DC_ERR_BAD_SHAPE: return "bad batch, L or direction";
+        case DC_ERR_NEGATIVE: return "negative cost or latency";
+        case DC_ERR_RANGE: return "L*dt + sum(xfer) + sum(comp) >= 2^52";
+        case DC_ERR_WORKSPACE: return "workspace missing or too small";
+        case DC_ERR_CUDA: return "CUDA runtime error";
+        case DC_ERR_BAD_CONFIG: return "profile generator config out of range";
+        case DC_ERR_INTERNAL: return "solver self-check failed";
+    }
+    return "unknown status";
+}
+
+dc_status dc_roof_int_probe(int32_t variant, int32_t blocks, int32_t threads, int64_t iters,
+                            uint32_t *sink, cudaStream_t stream)
+{
+    if (variant != 0 && variant != 1) return DC_ERR_BAD_SHAPE;
+    if (blocks < 1 || threads < 32 || threads > 1024 || threads % 32 || iters < 0 || iters % 4)
+        return DC_ERR_BAD_SHAPE;
+    if (!sink) return DC_ERR_NULL;
+    return dc::launch_roof(variant, blocks, threads, iters, sink, stream) == cudaSuccess
+               ? DC_OK
+               : DC_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,250 @@
+// Seeded synthetic profile generator (stand-in for the real-time profiler of
+// Sec. IV-A, which derives pt, fc, bc, gt and dt from a framework's profiler).
+//
+// One thread per (instance, layer) element; every value is a pure function of
+// (seed, global instance index, field, layer), so any sub-range of a batch can
+// be generated on its own. Integer-only on the device: SplitMix64 draws,
+// multiply-high uniform integers, piecewise-linear log-uniform knots built on the
+// host in double precision, and exact ceiling divisions (float reciprocal
+// estimate + integer remainder correction, no 64-bit divide in the common path).
+#include <cmath>
+
+#include "common.cuh"
+
+namespace dc {
+namespace {
+
+constexpr int kKnots = 512;
+constexpr int kFixedMax = 1024;
+
+struct GenParams {
+    int64_t batch, inst0;
+    uint64_t seed;
+    int32_t L, layer_mode, rate_dist, bw_dist, bwd_mult, bits;
+    int64_t rate_lo, rate_hi, bw_lo, bw_hi, dt_lo, dt_hi;
+    int64_t params_lo, params_hi, flops_lo, flops_hi;
+    int64_t rate_knots[kKnots + 1], bw_knots[kKnots + 1];
+    // per-layer tables: fixed params/FLOPs, or log-uniform knots of the draws
+    int64_t layer0[kFixedMax], layer1[kFixedMax];
+};
+static_assert(sizeof(GenParams) < 32000, "kernel parameter block limit");
+
+__device__ __forceinline__ uint64_t splitmix(uint64_t seed, uint64_t ctr)
+{
+    uint64_t z = seed + (ctr + 1) * 0x9e3779b97f4a7c15ull;
+    z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ull;
+    z = (z ^ (z >> 27)) * 0x94d049bb133111ebull;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint64_t counter(int64_t gi, int field, int layer)
+{
+    return (uint64_t(gi) << 20) | (uint64_t(field) << 12) | uint64_t(layer);
+}
+
+__device__ __forceinline__ int64_t uniform_int(int64_t lo, int64_t hi, uint64_t r)
+{
+    return lo + int64_t(__umul64hi(r, uint64_t(hi - lo) + 1u));
+}
+
+__device__ __forceinline__ int64_t loguniform(const int64_t *knots, uint64_t r)
+{
+    const int j = int(r >> 55);
+    const uint64_t f = (r >> 23) & 0xffffffffull;
+    const int64_t t0 = knots[j], t1 = knots[j + 1];
+    return t0 + int64_t((uint64_t(t1 - t0) * f) >> 32);
+}
+
+// ceil(a / d), exact, for 0 <= a < 2^62 and 1 <= d < 2^31. Three float
+// estimates of the quotient, each correcting the previous one's remainder,
+// leave |remainder| <= d + 1; two bounded integer steps finish it. The plain
+// 64-bit division is kept only as an unreachable safety net.
+__device__ __forceinline__ uint64_t ceil_div(uint64_t a, uint32_t d)
+{
+    const float rd = __frcp_rn(float(d));
+    uint64_t q = __float2ull_rz(__ull2float_rn(a) * rd);
+    int64_t r = int64_t(a - q * uint64_t(d));
+#pragma unroll
+    for (int it = 0; it < 2; ++it) {
+        q = uint64_t(int64_t(q) + __float2ll_rz(__ll2float_rn(r) * rd));
+        r = int64_t(a - q * uint64_t(d));
+    }
+#pragma unroll
+    for (int it = 0; it < 2; ++it) {
+        if (r < 0) {
+            --q;
+            r += d;
+        }
+        if (r >= int64_t(d)) {
+            ++q;
+            r -= d;
+        }
+    }
+    if (r < 0 || r >= int64_t(d)) {
+        q = a / d;
+        r = int64_t(a - q * d);
+    }
+    return q + (r != 0 ? 1u : 0u);
+}
+
+__global__ void __launch_bounds__(256)
+    gen_kernel(const __grid_constant__ GenParams g, int64_t *__restrict__ fc,
+               int64_t *__restrict__ pt, int64_t *__restrict__ bc, int64_t *__restrict__ gt,
+               int64_t *__restrict__ dt)
+{
+    __shared__ int64_t s_rate[kKnots + 1], s_bw[kKnots + 1];
+    __shared__ int64_t s_l0[kFixedMax], s_l1[kFixedMax];
+    const int L = g.L;
+    const int nl = g.layer_mode == DC_LAYERS_FIXED ? L : (g.layer_mode == DC_LAYERS_LOGUNIFORM ? kKnots + 1 : 0);
+    for (int j = threadIdx.x; j <= kKnots; j += blockDim.x) {
+        s_rate[j] = g.rate_knots[j];
+        s_bw[j] = g.bw_knots[j];
+    }
+    for (int j = threadIdx.x; j < nl; j += blockDim.x) {
+        s_l0[j] = g.layer0[j];
+        s_l1[j] = g.layer1[j];
+    }
+    __syncthreads();
+
+    const int64_t total = g.batch * L;
+    const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+    int64_t e = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= total) return;
+    // (i, l) of element e, advanced incrementally by the grid stride
+    int64_t i = e / L;
+    int l = int(e - i * L);
+    const int64_t di = stride / L;
+    const int dl = int(stride - di * L);
+    for (; e < total; e += stride) {
+        const int64_t gi = g.inst0 + i;
+        const uint64_t r_rate = splitmix(g.seed, counter(gi, 0, 0));
+        const uint64_t r_bw = splitmix(g.seed, counter(gi, 1, 0));
+        const int64_t rate = g.rate_dist == DC_DIST_LOGUNIFORM
+                                 ? loguniform(s_rate, r_rate)
+                                 : uniform_int(g.rate_lo, g.rate_hi, r_rate);
+        const int64_t bw = g.bw_dist == DC_DIST_LOGUNIFORM ? loguniform(s_bw, r_bw)
+                                                           : uniform_int(g.bw_lo, g.bw_hi, r_bw);
+        int64_t params, flops;
+        if (g.layer_mode == DC_LAYERS_FIXED) {
+            params = s_l0[l];
+            flops = s_l1[l];
+        } else {
+            const uint64_t rp = splitmix(g.seed, counter(gi, 3, l));
+            const uint64_t rf = splitmix(g.seed, counter(gi, 4, l));
+            if (g.layer_mode == DC_LAYERS_LOGUNIFORM) {
+                params = loguniform(s_l0, rp);
+                flops = loguniform(s_l1, rf);
+            } else {
+                params = uniform_int(g.params_lo, g.params_hi, rp);
+                flops = uniform_int(g.flops_lo, g.flops_hi, rf);
+            }
+        }
+        const uint64_t xfer =
+            ceil_div(uint64_t(g.bits) * 1000u * uint64_t(params), uint32_t(bw));
+        fc[e] = int64_t(ceil_div(uint64_t(flops), uint32_t(rate)));
+        bc[e] = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), uint32_t(rate)));
+        pt[e] = int64_t(xfer);
+        gt[e] = int64_t(xfer);
+        if (l == 0) dt[i] = uniform_int(g.dt_lo, g.dt_hi, splitmix(g.seed, counter(gi, 2, 0)));
+        i += di;
+        l += dl;
+        if (l >= L) {
+            l -= L;
+            ++i;
+        }
+    }
+}
+
+int64_t knot(int64_t lo, int64_t hi, int j)
+{
+    if (j <= 0) return lo;
+    if (j >= kKnots) return hi;
+    const double x = double(j) / 512.0;
+    const double y = std::log(double(hi) / double(lo));
+    return int64_t(std::llround(double(lo) * std::exp(x * y)));
+}
+
+void knots(int64_t lo, int64_t hi, int64_t *out)
+{
+    for (int j = 0; j <= kKnots; ++j) out[j] = knot(lo, hi, j);
+}
+
+bool in_range(int64_t lo, int64_t hi, int64_t min_lo, int64_t max_hi)
+{
+    return lo >= min_lo && lo <= hi && hi <= max_hi;
+}
+
+}  // namespace
+
+dc_status check_profile_cfg(const dc_profile_cfg *c)
+{
+    const int64_t cap = int64_t(1) << 40, rcap = (int64_t(1) << 31) - 1;
+    if (c->L < 1 || c->L > DC_L_MAX || c->batch < 0 || c->inst0 < 0) return DC_ERR_BAD_CONFIG;
+    if (c->inst0 + c->batch > (int64_t(1) << 44)) return DC_ERR_BAD_CONFIG;
+    if (c->bwd_flops_mult < 1 || c->bwd_flops_mult > 16) return DC_ERR_BAD_CONFIG;
+    if (c->bits_per_param < 1 || c->bits_per_param > 64) return DC_ERR_BAD_CONFIG;
+    if (!in_range(c->rate_lo, c->rate_hi, 1, rcap) || !in_range(c->bw_lo, c->bw_hi, 1, rcap))
+        return DC_ERR_BAD_CONFIG;
+    if (!in_range(c->dt_lo, c->dt_hi, 0, cap)) return DC_ERR_BAD_CONFIG;
+    if (c->rate_dist < 0 || c->rate_dist > 1 || c->bw_dist < 0 || c->bw_dist > 1)
+        return DC_ERR_BAD_CONFIG;
+    if (c->layer_mode == DC_LAYERS_FIXED) {
+        if (c->L > kFixedMax) return DC_ERR_BAD_CONFIG;
+        if (!c->fixed_params || !c->fixed_flops) return DC_ERR_NULL;
+        for (int l = 0; l < c->L; ++l)
+            if (!in_range(c->fixed_params[l], c->fixed_params[l], 0, cap) ||
+                !in_range(c->fixed_flops[l], c->fixed_flops[l], 0, cap))
+                return DC_ERR_BAD_CONFIG;
+    } else if (c->layer_mode == DC_LAYERS_UNIFORM || c->layer_mode == DC_LAYERS_LOGUNIFORM) {
+        const int64_t min_lo = c->layer_mode == DC_LAYERS_LOGUNIFORM ? 1 : 0;
+        if (!in_range(c->params_lo, c->params_hi, min_lo, cap) ||
+            !in_range(c->flops_lo, c->flops_hi, min_lo, cap))
+            return DC_ERR_BAD_CONFIG;
+    } else {
+        return DC_ERR_BAD_CONFIG;
+    }
+    return DC_OK;
+}
+
+cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_t *bc,
+                       int64_t *gt, int64_t *dt, cudaStream_t stream)
+{
+    static thread_local GenParams g;  // 25 KB: kept off the caller's stack
+    g.batch = c->batch;
+    g.inst0 = c->inst0;
+    g.seed = c->seed;
+    g.L = c->L;
+    g.layer_mode = c->layer_mode;
+    g.rate_dist = c->rate_dist;
+    g.bw_dist = c->bw_dist;
+    g.bwd_mult = c->bwd_flops_mult;
+    g.bits = c->bits_per_param;
+    g.rate_lo = c->rate_lo;
+    g.rate_hi = c->rate_hi;
+    g.bw_lo = c->bw_lo;
+    g.bw_hi = c->bw_hi;
+    g.dt_lo = c->dt_lo;
+    g.dt_hi = c->dt_hi;
+    g.params_lo = c->params_lo;
+    g.params_hi = c->params_hi;
+    g.flops_lo = c->flops_lo;
+    g.flops_hi = c->flops_hi;
+    if (c->rate_dist == DC_DIST_LOGUNIFORM) knots(c->rate_lo, c->rate_hi, g.rate_knots);
+    if (c->bw_dist == DC_DIST_LOGUNIFORM) knots(c->bw_lo, c->bw_hi, g.bw_knots);
+    if (c->layer_mode == DC_LAYERS_FIXED) {
+        for (int l = 0; l < c->L; ++l) {
+            g.layer0[l] = c->fixed_params[l];
+            g.layer1[l] = c->fixed_flops[l];
+        }
+    } else if (c->layer_mode == DC_LAYERS_LOGUNIFORM) {
+        knots(c->params_lo, c->params_hi, g.layer0);
+        knots(c->flops_lo, c->flops_hi, g.layer1);
+    }
+    const int64_t total = c->batch * c->L;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    gen_kernel<<<unsigned(blocks), 256, 0, stream>>>(g, fc, pt, bc, gt, dt);
+    return cudaGetLastError();
+}
+
+}  // namespace dc

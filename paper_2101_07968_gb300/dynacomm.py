@@ -1,0 +1,241 @@
+"""ctypes binding of libdynacomm.so (the C ABI in include/dynacomm.h).
+
+The ``dc_*`` functions keep the C names and argument order and only marshal
+arguments: torch tensors (or raw integer addresses) become device pointers and
+the stream defaults to torch's current CUDA stream. Every step of the
+scheduling path runs in the library's kernels; there is no CPU fallback, and
+loading fails loudly when the library has not been built.
+
+The convenience wrappers at the bottom (``profile_gen``, ``schedule``,
+``eval_timeline``) allocate output tensors with torch and call the ``dc_*``
+functions.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libdynacomm.so")
+
+DC_OK, DC_ERR_NULL, DC_ERR_BAD_SHAPE, DC_ERR_NEGATIVE, DC_ERR_RANGE = 0, 1, 2, 3, 4
+DC_ERR_WORKSPACE, DC_ERR_CUDA, DC_ERR_BAD_CONFIG, DC_ERR_INTERNAL = 5, 6, 7, 8
+DC_L_MAX = 4096
+FWD, BWD = 0, 1
+
+
+class DynaCommError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {dc_status_string(status)} (status {status})")
+        self.status = status
+
+
+class dc_profile_cfg(ctypes.Structure):
+    _fields_ = [
+        ("L", ctypes.c_int32), ("layer_mode", ctypes.c_int32),
+        ("batch", ctypes.c_int64), ("inst0", ctypes.c_int64), ("seed", ctypes.c_uint64),
+        ("fixed_params", ctypes.POINTER(ctypes.c_int64)),
+        ("fixed_flops", ctypes.POINTER(ctypes.c_int64)),
+        ("params_lo", ctypes.c_int64), ("params_hi", ctypes.c_int64),
+        ("flops_lo", ctypes.c_int64), ("flops_hi", ctypes.c_int64),
+        ("rate_dist", ctypes.c_int32), ("bw_dist", ctypes.c_int32),
+        ("rate_lo", ctypes.c_int64), ("rate_hi", ctypes.c_int64),
+        ("bw_lo", ctypes.c_int64), ("bw_hi", ctypes.c_int64),
+        ("dt_lo", ctypes.c_int64), ("dt_hi", ctypes.c_int64),
+        ("bwd_flops_mult", ctypes.c_int32), ("bits_per_param", ctypes.c_int32),
+    ]
+
+
+_lib = None
+
+# name -> (restype, argtypes); the exported C ABI
+_VP, _I32, _I64, _SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+_SIGNATURES = {
+    "dc_profile_gen": (_I32, [ctypes.POINTER(dc_profile_cfg), _VP, _VP, _VP, _VP, _VP, _VP]),
+    "dc_schedule_workspace_bytes": (_SZ, [_I64, _I32]),
+    "dc_schedule_forward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                         _SZ, _VP]),
+    "dc_schedule_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                          _SZ, _VP]),
+    "dc_eval_timeline_batch": (_I32, [_I64, _I32, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
+    "dc_status_string": (ctypes.c_char_p, [_I32]),
+    "dc_roof_int_probe": (_I32, [_I32, _I32, _I32, _I64, _VP, _VP]),
+}
+
+
+def lib():
+    """Load libdynacomm.so (raises if it is missing: build it first)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(
+                f"{LIB_PATH} is missing: build it with `python -m paper_2101_07968_gb300.build`")
+        l = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(l, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = l
+    return _lib
+
+
+def exported_names():
+    return list(_SIGNATURES)
+
+
+# ------------------------------------------------------------- marshalling
+def _ptr(x) -> Optional[int]:
+    """torch tensor -> device address (must be CUDA); int -> itself; None -> NULL."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if not x.is_cuda:
+        raise ValueError("device tensor expected (the library takes device pointers)")
+    if not x.is_contiguous():
+        raise ValueError("contiguous tensor expected")
+    return x.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        if not torch.cuda.is_available():
+            return None
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(st: int, what: str):
+    if st != DC_OK:
+        raise DynaCommError(st, what)
+    return st
+
+
+# -------------------------------------------------------------- C ABI names
+def dc_status_string(status: int) -> str:
+    return lib().dc_status_string(int(status)).decode()
+
+
+def dc_schedule_workspace_bytes(batch: int, L: int) -> int:
+    return int(lib().dc_schedule_workspace_bytes(int(batch), int(L)))
+
+
+def make_cfg(cfg: dict, keep: list) -> dc_profile_cfg:
+    """dict (see workloads.config) -> dc_profile_cfg; `keep` holds host arrays alive."""
+    c = dc_profile_cfg()
+    c.L = int(cfg["L"])
+    c.layer_mode = int(cfg["layer_mode"])
+    c.batch = int(cfg["batch"])
+    c.inst0 = int(cfg.get("inst0", 0))
+    c.seed = int(cfg["seed"])
+    if int(cfg["layer_mode"]) == 0:
+        import numpy as np
+        fp = np.ascontiguousarray(cfg["fixed_params"], dtype=np.int64)
+        ff = np.ascontiguousarray(cfg["fixed_flops"], dtype=np.int64)
+        keep += [fp, ff]
+        c.fixed_params = fp.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
+        c.fixed_flops = ff.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
+    for k in ("params_lo", "params_hi", "flops_lo", "flops_hi", "rate_lo", "rate_hi",
+              "bw_lo", "bw_hi", "dt_lo", "dt_hi"):
+        setattr(c, k, int(cfg.get(k, 0)))
+    c.rate_dist = int(cfg["rate_dist"])
+    c.bw_dist = int(cfg["bw_dist"])
+    c.bwd_flops_mult = int(cfg.get("bwd_flops_mult", 2))
+    c.bits_per_param = int(cfg.get("bits_per_param", 32))
+    return c
+
+
+def dc_profile_gen(cfg, fc, pt, bc, gt, dt, stream=None) -> int:
+    keep: list = []
+    c = cfg if isinstance(cfg, dc_profile_cfg) else make_cfg(cfg, keep)
+    return int(lib().dc_profile_gen(ctypes.byref(c), _ptr(fc), _ptr(pt), _ptr(bc), _ptr(gt),
+                                    _ptr(dt), _stream(stream)))
+
+
+def dc_schedule_forward_batch(batch, L, fc, pt, dt, makespan, bits, nseg, status, workspace,
+                              workspace_bytes, stream=None) -> int:
+    return int(lib().dc_schedule_forward_batch(
+        int(batch), int(L), _ptr(fc), _ptr(pt), _ptr(dt), _ptr(makespan), _ptr(bits),
+        _ptr(nseg), _ptr(status), _ptr(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def dc_schedule_backward_batch(batch, L, bc, gt, dt, makespan, bits, nseg, status, workspace,
+                               workspace_bytes, stream=None) -> int:
+    return int(lib().dc_schedule_backward_batch(
+        int(batch), int(L), _ptr(bc), _ptr(gt), _ptr(dt), _ptr(makespan), _ptr(bits),
+        _ptr(nseg), _ptr(status), _ptr(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def dc_eval_timeline_batch(batch, L, direction, comp, xfer, dt, bits, makespan,
+                           stream=None) -> int:
+    return int(lib().dc_eval_timeline_batch(
+        int(batch), int(L), int(direction), _ptr(comp), _ptr(xfer), _ptr(dt), _ptr(bits),
+        _ptr(makespan), _stream(stream)))
+
+
+def dc_roof_int_probe(variant, blocks, threads, iters, sink, stream=None) -> int:
+    return int(lib().dc_roof_int_probe(int(variant), int(blocks), int(threads), int(iters),
+                                       _ptr(sink), _stream(stream)))
+
+
+# ------------------------------------------------------------ conveniences
+def words(L: int) -> int:
+    return (L - 1 + 31) // 32
+
+
+def profile_gen(cfg: dict, device="cuda", stream=None) -> dict:
+    """Allocate and fill fc, pt, bc, gt [batch, L] and dt [batch] (int64, device)."""
+    import torch
+    B, L = int(cfg["batch"]), int(cfg["L"])
+    out = {k: torch.empty((B, L), dtype=torch.int64, device=device)
+           for k in ("fc", "pt", "bc", "gt")}
+    out["dt"] = torch.empty(B, dtype=torch.int64, device=device)
+    _check(dc_profile_gen(cfg, out["fc"], out["pt"], out["bc"], out["gt"], out["dt"], stream),
+           "dc_profile_gen")
+    return out
+
+
+class Scheduler:
+    """Owns a reusable workspace and output buffers for one (batch, L)."""
+
+    def __init__(self, batch: int, L: int, device="cuda"):
+        import torch
+        self.batch, self.L, self.W = int(batch), int(L), words(L)
+        self.ws_bytes = dc_schedule_workspace_bytes(batch, L)
+        self.workspace = torch.empty(max(self.ws_bytes, 1), dtype=torch.uint8, device=device)
+        self.out = {}
+        for d in (FWD, BWD):
+            self.out[d] = dict(
+                makespan=torch.empty(self.batch, dtype=torch.int64, device=device),
+                bits=torch.empty((self.batch, max(self.W, 1)), dtype=torch.int32,
+                                 device=device),
+                nseg=torch.empty(self.batch, dtype=torch.int32, device=device),
+                status=torch.empty(self.batch, dtype=torch.int32, device=device))
+
+    def run(self, direction: int, comp, xfer, dt, stream=None) -> dict:
+        o = self.out[direction]
+        fn = dc_schedule_forward_batch if direction == FWD else dc_schedule_backward_batch
+        _check(fn(self.batch, self.L, comp, xfer, dt, o["makespan"], o["bits"], o["nseg"],
+                  o["status"], self.workspace, self.ws_bytes, stream),
+               "dc_schedule_forward_batch" if direction == FWD else "dc_schedule_backward_batch")
+        return o
+
+
+def schedule(direction: int, comp, xfer, dt, stream=None) -> dict:
+    """One direction for a batch: makespan, bits (int32 view of uint32 words), nseg, status."""
+    B, L = comp.shape
+    s = Scheduler(B, L, device=comp.device)
+    return s.run(direction, comp, xfer, dt, stream)
+
+
+def eval_timeline(direction: int, comp, xfer, dt, bits, stream=None):
+    import torch
+    B, L = comp.shape
+    out = torch.empty(B, dtype=torch.int64, device=comp.device)
+    _check(dc_eval_timeline_batch(B, L, direction, comp, xfer, dt, bits, out, stream),
+           "dc_eval_timeline_batch")
+    return out

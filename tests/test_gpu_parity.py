@@ -1,0 +1,239 @@
+"""GPU (sm_103a) path against the CPU oracle, element by element, through the C ABI.
+
+Integer work, so the bar is bit-exact: makespan, every decision word, nseg and
+status for the DP; every int64 of the generated profiles; every makespan of the
+timeline replay. Inputs are seeded and synthetic; every expected value comes
+from the oracle.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2101_07968_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+FWD, BWD = 0, 1
+NTHREADS = os.cpu_count() or 1
+
+
+@pytest.fixture(scope="module")
+def dc():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2101_07968_gb300 import build, dynacomm
+    build.build()
+    dynacomm.lib()
+    return dynacomm
+
+
+def _dev(a):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _gpu_schedule(dc, direction, comp, xfer, dt):
+    import torch
+    B, L = comp.shape
+    out = dc.schedule(direction, _dev(comp), _dev(xfer), _dev(dt))
+    torch.cuda.synchronize()
+    W = dc.words(L)
+    res = {k: v.cpu().numpy() for k, v in out.items()}
+    res["bits"] = res["bits"].view(np.uint32)[:, :W] if W else np.zeros((B, 0), np.uint32)
+    return res
+
+
+def _assert_same(got, exp, label=""):
+    for key in ("status", "makespan", "nseg", "bits"):
+        g, e = got[key], exp[key]
+        if key == "bits":
+            g = g.reshape(e.shape)
+        bad = np.nonzero(g != e)[0] if g.ndim == 1 else np.nonzero((g != e).any(axis=1))[0]
+        assert bad.size == 0, (f"{label} {key}: {bad.size} mismatches, first at {bad[0]}: "
+                               f"gpu={g[bad[0]]} oracle={e[bad[0]]}")
+
+
+def _check_direction(dc, direction, comp, xfer, dt, label=""):
+    got = _gpu_schedule(dc, direction, comp, xfer, dt)
+    exp = oracle.schedule_batch(direction, comp, xfer, dt, nthreads=NTHREADS)
+    _assert_same(got, exp, label)
+    return got
+
+
+# ------------------------------------------------------------------ DP parity
+SMALL_LS = list(range(1, 21)) + [31, 32, 33, 40, 54, 63, 64, 65, 96, 130]
+
+
+@pytest.mark.parametrize("L", SMALL_LS)
+@pytest.mark.parametrize("kind", ["tie", "uni", "skew"])
+def test_dp_random_parity(dc, L, kind):
+    """Several tiles and a ragged tail for every kernel variant and width."""
+    B = {True: 700, False: 150}[L <= 20] + 13
+    gen = {"tie": wl.tie_heavy_instances, "uni": wl.random_instances,
+           "skew": wl.skewed_instances}[kind]
+    comp, xfer, dt = gen(1000 * L + len(kind), B, L)
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
+
+
+@pytest.mark.parametrize("L", [1, 2, 8, 16, 17, 54, 70])
+def test_dp_wide_values_parity(dc, L):
+    """Instances whose bound exceeds 2^32 need 64-bit arithmetic; mix them with
+    32-bit ones so both paths (and the work list) run in one call."""
+    B = 640 + 7
+    comp, xfer, dt = wl.skewed_instances(77 + L, B, L)
+    rng = np.random.default_rng(L)
+    wide = rng.random(B) < 0.3
+    scale = rng.integers(1 << 26, 1 << 36, size=(B, 1))
+    comp[wide] = comp[wide] * 3 + (scale[wide] * rng.random((wide.sum(), L))).astype(np.int64)
+    xfer[wide] = xfer[wide] + (scale[wide] * rng.random((wide.sum(), L))).astype(np.int64)
+    dt[wide[:]] += rng.integers(0, 1 << 30, size=wide.sum())
+    bound = L * dt + comp.sum(1) + xfer.sum(1)
+    assert (bound[wide] > 2**32).any() and (bound < 2**52).all()
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, f"wide L={L} dir={d}")
+
+
+@pytest.mark.parametrize("L", [8, 16, 54, 100])
+def test_dp_status_faults_per_instance(dc, L):
+    B = 300
+    comp, xfer, dt = wl.random_instances(5 + L, B, L, 0, 100_000, 0, 10_000)
+    comp[3, L - 1] = -5
+    xfer[10, 0] = -1
+    dt[20] = -7
+    xfer[30, L // 2] = 1 << 52                       # one value alone too big
+    comp[40, :] = (1 << 52) // L                      # sum too big
+    dt[50] = 1 << 51                                  # L * dt too big (L >= 2)
+    for d in (FWD, BWD):
+        got = _check_direction(dc, d, comp, xfer, dt, f"faults L={L} dir={d}")
+        assert list(got["status"][[3, 10, 20, 30, 40, 50]]) == [3, 3, 3, 4, 4, 4]
+        assert (got["status"][[0, 1, 2, 4, 299]] == 0).all()
+
+
+def test_dp_batch_zero_and_single(dc):
+    import torch
+    ws = torch.empty(4096, dtype=torch.uint8, device="cuda")
+    z = torch.empty(0, dtype=torch.int64, device="cuda")
+    assert dc.dc_schedule_forward_batch(0, 8, z, z, z, z, z, None, None, ws, 4096) == dc.DC_OK
+    comp, xfer, dt = wl.random_instances(3, 1, 1, 0, 50, 0, 50)
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, "batch=1 L=1")
+
+
+def test_dp_maximum_L(dc):
+    """L = 4096 (the largest the ABI takes): the backward optimum equals the 1-D
+    recurrence, both decisions replay to their makespans, and neither is worse
+    than layer-by-layer or sequential."""
+    L, B = 4096, 2
+    comp, xfer, dt = wl.random_instances(9, B, L, 0, 5_000, 0, 50_000)
+    for d in (FWD, BWD):
+        got = _gpu_schedule(dc, d, comp, xfer, dt)
+        assert (got["status"] == 0).all()
+        rep = oracle.replay_batch(d, comp, xfer, dt, got["bits"], nthreads=2)
+        assert np.array_equal(rep, got["makespan"])
+        seq = np.zeros((B, dc.words(L)), np.uint32)
+        lbl = oracle.replay_batch(d, comp, xfer, dt, np.full_like(seq, 0xFFFFFFFF) & _mask(L))
+        assert (got["makespan"] <= oracle.replay_batch(d, comp, xfer, dt, seq)).all()
+        assert (got["makespan"] <= lbl).all()
+        assert (got["nseg"] == 1 + np.unpackbits(got["bits"].view(np.uint8), axis=1).sum(1)).all()
+        if d == BWD:
+            for i in range(B):
+                assert got["makespan"][i] == oracle.dp_backward_1d(comp[i], xfer[i], dt[i])
+
+
+def _mask(L):
+    W = (L - 1 + 31) // 32
+    m = np.zeros(W, np.uint32)
+    for l in range(L - 1):
+        m[l // 32] |= np.uint32(1 << (l % 32))
+    return m
+
+
+# ------------------------------------------------------- generator parity
+@pytest.mark.parametrize("name", wl.CONFIG_NAMES)
+def test_profile_gen_bitwise(dc, name):
+    """Full batch of every configuration, every int64 equal to the oracle's."""
+    import torch
+    cfg = wl.config(name)
+    got = dc.profile_gen(cfg)
+    torch.cuda.synchronize()
+    exp = oracle.profile_gen(cfg)
+    for k in ("fc", "pt", "bc", "gt", "dt"):
+        g = got[k].cpu().numpy()
+        bad = np.nonzero((g != exp[k]).reshape(len(g), -1).any(axis=1))[0]
+        assert bad.size == 0, f"{name}.{k}: {bad.size} rows differ, first {bad[:3]}"
+
+
+def test_profile_gen_offset_and_ragged(dc):
+    import torch
+    cfg = wl.with_batch(wl.config("deepchain"), 37, inst0=123_456)
+    cfg["L"] = 77
+    got = dc.profile_gen(cfg)
+    torch.cuda.synchronize()
+    exp = oracle.profile_gen(cfg)
+    for k in ("fc", "pt", "bc", "gt", "dt"):
+        assert np.array_equal(got[k].cpu().numpy(), exp[k])
+
+
+# -------------------------------------------------------- timeline parity
+@pytest.mark.parametrize("L", [1, 2, 7, 16, 32, 33, 54, 65, 1024])
+def test_eval_timeline_random_decisions(dc, L):
+    import torch
+    B = 500 + 3
+    comp, xfer, dt = wl.skewed_instances(31 * L, B, L)
+    comp[5, 0] = -1
+    dt[9] = 1 << 52
+    bits = wl.random_decisions(L, B, L, density=0.3)
+    for d in (FWD, BWD):
+        got = dc.eval_timeline(d, _dev(comp), _dev(xfer), _dev(dt),
+                               _dev(bits.view(np.int32)) if bits.size else None)
+        torch.cuda.synchronize()
+        exp = oracle.replay_batch(d, comp, xfer, dt, bits, nthreads=NTHREADS)
+        assert np.array_equal(got.cpu().numpy(), exp)
+
+
+# ---------------------------------------------- full-size configurations
+def _config_parity(dc, name, sample=None):
+    cfg = wl.config(name)
+    prof = oracle.profile_gen(cfg)
+    for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+        got = _gpu_schedule(dc, d, prof[c], prof[x], prof["dt"])
+        if sample is None:
+            exp = oracle.schedule_batch(d, prof[c], prof[x], prof["dt"], nthreads=NTHREADS)
+            _assert_same(got, exp, f"{name} dir={d}")
+        else:
+            idx = np.asarray(sample)
+            exp = oracle.schedule_batch(d, prof[c][idx], prof[x][idx], prof["dt"][idx],
+                                        nthreads=NTHREADS)
+            sub = {k: v[idx] for k, v in got.items()}
+            _assert_same(sub, exp, f"{name} dir={d} sample")
+            # every instance: the decision replays to the makespan
+            rep = oracle.replay_batch(d, prof[c], prof[x], prof["dt"], got["bits"],
+                                      nthreads=NTHREADS)
+            assert np.array_equal(rep, got["makespan"])
+            if d == BWD:
+                for i in idx[:64]:
+                    assert got["makespan"][i] == oracle.dp_backward_1d(
+                        prof[c][i], prof[x][i], prof["dt"][i])
+
+
+@pytest.mark.parametrize("name", ["tiny", "alexnet", "vgg16", "resnet50"])
+def test_config_full_batch_parity(dc, name):
+    _config_parity(dc, name)
+
+
+def test_config_deepchain_sampled_parity(dc):
+    rng = np.random.default_rng(4)
+    sample = np.concatenate([[0, 1, 16383], rng.integers(0, 16384, size=5)])
+    _config_parity(dc, "deepchain", sample=sample)
+
+
+def test_roof_probe_runs(dc):
+    import torch
+    sink = torch.empty(152 * 256, dtype=torch.int32, device="cuda")
+    for v in (0, 1):
+        assert dc.dc_roof_int_probe(v, 152, 256, 64, sink) == dc.DC_OK
+    torch.cuda.synchronize()
