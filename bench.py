@@ -149,6 +149,8 @@ def run_reference(args):
     import oracle
     oracle.build()
     cfg = wl.config(args.workload)
+    if args.batch:
+        cfg = wl.with_batch(cfg, args.batch)
     cores = os.cpu_count() or 1
     sample = min(cfg["batch"], CPU_SAMPLE[args.workload])
     for _ in range(args.warmup):
@@ -195,6 +197,8 @@ def run_ours(args):
     dev = torch.device("cuda", torch.cuda.current_device())
 
     base = wl.config(args.workload)
+    if args.batch:
+        base = wl.with_batch(base, args.batch)
     B, L = base["batch"], base["L"]
     cfg = wl.with_batch(base, B, inst0=rank * B)  # distinct instances per rank
     W = dc.words(L)
@@ -273,7 +277,8 @@ def run_ours(args):
         roof[variant] = roof_blocks * roof_threads * roof_iters * 8 / (r0.elapsed_time(r1) * 1e-3)
 
     # ---- end to end through the public API with host buffers
-    e2e = run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world)
+    e2e = None if args.no_e2e else run_e2e(dc, torch, prof, sched, B, L, W, dev, args,
+                                           barrier, world)
 
     # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
     cpu = None
@@ -410,7 +415,11 @@ def main(argv=None):
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", choices=list(wl.CONFIG_NAMES), default="vgg16")
+    p.add_argument("--batch", type=int, default=0,
+                   help="instances per GPU (default: the workload's batch); for profiling "
+                        "small cases")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
     args = p.parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)

@@ -10,188 +10,136 @@
 //
 // Design (GB300):
 //  * one instance per thread, 32 instances per warp, no inter-thread traffic in
-//    the fill; the whole DP runs in registers with compile-time indices;
-//  * values are 32-bit whenever the instance bound L*dt + sum(xfer) + sum(comp)
-//    is below 2^32 - 1: every DP value and every candidate lies in
-//    [0, bound], so the 32-bit fill is exact. Other instances go to a work
-//    list solved in 64-bit by the group kernel;
+//    the fill; the DP column lives in registers with compile-time indices;
 //  * the fill keeps only the minimum VALUE per cell (max, subtract, min per
-//    transition). Each finished cell is stored to the lane's slice of shared
-//    memory; the traceback then recovers Path[m][n] as the lowest k whose
-//    candidate equals the cell, which is exactly the k Algorithm 3/4 keeps
-//    with its strict-improvement test;
-//  * the warp's rows are loaded with coalesced 64-bit loads into a padded shared
-//    buffer (odd row stride: no bank conflicts when each lane reads its row).
+//    transition: two integer-ALU-pipe operations, the subtraction can issue on
+//    the FMA pipe). Finished cells go to the lane's slice of shared memory; the
+//    traceback recovers Path[m][n] as the lowest k whose candidate equals the
+//    cell, which is the k Algorithm 3/4 keeps with its strict-improvement test.
+//    Column 1 (X[m][1] = R(m,1) + S[m] + c) and column L (one cell, the
+//    makespan) are not stored;
+//  * 32-bit values whenever the instance bound L*dt + sum(xfer) + sum(comp) is
+//    below 2^32 - 1: every DP value and candidate lies in [0, bound], so the
+//    32-bit fill is exact. Other instances are appended to a work list that a
+//    64-bit instantiation of the same kernel solves afterwards;
+//  * persistent warps: each warp walks 32-instance tiles; while it solves one
+//    tile, the next tile's rows stream into a padded shared buffer with
+//    cp.async (coalesced 8-byte copies, odd row stride so that every lane reads
+//    its own row without bank conflicts).
 #include "common.cuh"
 
 namespace dc {
 namespace {
 
-template <int L>
+template <int L, typename T>
 struct Small {
-    static constexpr int kCells = L * (L + 1) / 2;
-    static constexpr int kOffS = kCells;          // per-lane word offset of S[0..L]
-    static constexpr int kOffR = kCells + L + 1;  // per-lane word offset of R[0..L]
-    static constexpr int kLaneWords = kCells + 2 * (L + 1);
-    static constexpr int kStride = (L % 2 == 0) ? L + 1 : L;  // staging stride, int64 units
-    static constexpr int kStageWords = 2 * 32 * kStride * 2;
-    static constexpr int kWarpWords =
-        (32 * kLaneWords > kStageWords) ? 32 * kLaneWords : kStageWords;
-    static constexpr int kWarpBytes = kWarpWords * 4;
-    static constexpr int kWarps0 = (48 * 1024) / kWarpBytes;
-    static constexpr int kWarps = kWarps0 < 1 ? 1 : (kWarps0 > 8 ? 8 : kWarps0);
-    static constexpr int kThreads = 32 * kWarps;
-    static constexpr int kSmemBytes = kWarps * kWarpBytes;
+    static constexpr int kCells = L >= 2 ? L * (L + 1) / 2 - L - 1 : 0;  // columns 2..L-1
+    static constexpr int kW = sizeof(T) / 4;                            // words per value
+    static constexpr int kOffS = kCells;                                // S[0..L]
+    static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
+    static constexpr int kLaneVals = kCells + 2 * (L + 1);
+    static constexpr int kStride = (L % 2 == 0) ? L + 1 : L;  // staging row stride (int64, odd)
+    static constexpr int kStageBytes = 2 * 32 * kStride * 8;   // comp + xfer rows of a tile
+    static constexpr int kTableBytes = 32 * kLaneVals * int(sizeof(T));
+    static constexpr int kWarpBytes = kStageBytes + kTableBytes;
 };
 
-__host__ __device__ constexpr int cell_of(int L, int m, int n) { return (n - 1) * L - (n - 1) * (n - 2) / 2 + (m - n); }
-
-// The 32-bit fill. lw = this lane's words in shared memory (word w at lw[32*w]).
-template <int L, bool FWD>
-__device__ __forceinline__ void fill32(const uint32_t (&S)[L + 1], const uint32_t (&Rb)[L + 1],
-                                       uint32_t dtv, uint32_t c, uint32_t *lw, uint32_t &T,
-                                       int &s)
+// index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
+__host__ __device__ constexpr int cell2(int L, int m, int n)
 {
-    uint32_t col[L + 1];
-    // column n = 1: the only finite predecessor is X[0][0] = 0 and S[0] = 0
+    return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
+}
+
+template <typename T>
+__device__ __forceinline__ T lds(const T *lane_base, int v) { return lane_base[32 * v]; }
+
+// The fill. lw = this lane's values in shared memory (value v at lw[32*v]).
+template <int L, bool FWD, typename T>
+__device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], T dtv, T c,
+                                     T *lw, T &best_T, int &best_s)
+{
+    T col[L + 1];
 #pragma unroll
-    for (int m = 1; m <= L; ++m) {
-        const uint32_t R = FWD ? dtv + Rb[m] : Rb[m];
-        col[m] = R + S[m] + c;
-        lw[32 * cell_of(L, m, 1)] = col[m];
-    }
-    T = col[L];
-    s = 1;
+    for (int m = 1; m <= L; ++m) col[m] = T((FWD ? T(dtv + Rb[m]) : Rb[m]) + S[m] + c);
+    best_T = col[L];
+    best_s = 1;
 #pragma unroll
     for (int n = 2; n <= L; ++n) {
         // rows in descending order so column n overwrites column n-1 in place:
         // row m reads rows k < m, which still hold column n-1.
 #pragma unroll
         for (int m = L; m >= n; --m) {
-            const uint32_t R = FWD ? uint32_t(n) * dtv + Rb[m] : Rb[m];
-            uint32_t best = dmax(col[n - 1], R) - S[n - 1];
+            const T R = FWD ? T(T(n) * dtv + Rb[m]) : Rb[m];
+            constexpr int kMax = L;
+            T cand[kMax];
+            const int cnt = m - n + 1;  // k = n-1 .. m-1
 #pragma unroll
-            for (int k = n; k < m; ++k) best = dmin(best, dmax(col[k], R) - S[k]);
-            col[m] = best + S[m] + c;
-            lw[32 * cell_of(L, m, n)] = col[m];
+            for (int j = 0; j < cnt; ++j) cand[j] = T(dmax(col[n - 1 + j], R) - S[n - 1 + j]);
+#pragma unroll
+            for (int w = 1; w < cnt; w *= 2) {
+#pragma unroll
+                for (int j = 0; j + w < cnt; j += 2 * w) cand[j] = dmin(cand[j], cand[j + w]);
+            }
+            col[m] = T(cand[0] + S[m] + c);
+            if (n <= L - 1) lw[32 * cell2(L, m, n)] = col[m];
         }
-        if (col[L] < T) {  // strict: the lowest n wins ties
-            T = col[L];
-            s = n;
+        if (col[L] < best_T) {  // strict: the lowest n wins ties
+            best_T = col[L];
+            best_s = n;
         }
     }
 }
 
-template <int L, bool FWD>
-__global__ void __launch_bounds__(Small<L>::kThreads)
-    small_kernel(int64_t batch, const int64_t *__restrict__ comp,
-                 const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
-                 int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,
-                 int32_t *__restrict__ nseg, int32_t *__restrict__ status,
-                 uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list)
+// X[k][n-1] during the traceback: column 1 from S and R, others from the table.
+template <int L, bool FWD, typename T>
+__device__ __forceinline__ T prev_cell(const T *lw, int k, int nm1, T dtv, T c)
 {
-    using K = Small<L>;
+    using K = Small<L, T>;
+    if (nm1 == 1) {
+        const T r = lds(lw, K::kOffR + k);
+        return T((FWD ? T(dtv + r) : r) + lds(lw, K::kOffS + k) + c);
+    }
+    return lds(lw, cell2(L, k, nm1));
+}
+
+// Solve one instance (row data already reduced to 64-bit prefix sums in
+// processing order) and write its outputs.
+template <int L, bool FWD, typename T>
+__device__ __forceinline__ void solve(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+                                      int64_t dti, T *lw, int64_t i, int64_t *makespan,
+                                      uint32_t *bits, int32_t *nseg, int32_t *status)
+{
+    using K = Small<L, T>;
     constexpr int W = (L - 1 + 31) / 32;
-    extern __shared__ __align__(16) uint32_t smem[];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    uint32_t *region = smem + warp * K::kWarpWords;
-    const int64_t base = (int64_t(blockIdx.x) * K::kWarps + warp) * 32;
-    if (base >= batch) return;  // warp-uniform
-    const int rows = int(batch - base < 32 ? batch - base : 32);
-    const int64_t i = base + lane;
-    const bool active = lane < rows;
-
-    // ---- coalesced staging of the warp's 32 rows of comp and xfer
-    int64_t *stC = reinterpret_cast<int64_t *>(region);
-    int64_t *stX = stC + 32 * K::kStride;
-    {
-        const int64_t *gC = comp + base * L;
-        const int64_t *gX = xfer + base * L;
-        const int nel = rows * L;
-        for (int e = lane; e < nel; e += 32) {
-            const int r = e / L, cidx = e - r * L;
-            stC[r * K::kStride + cidx] = __ldg(gC + e);
-            stX[r * K::kStride + cidx] = __ldg(gX + e);
-        }
-    }
-    const int64_t dti = active ? __ldg(dt + i) : 0;
-    __syncwarp();
-
-    // ---- own row, processing order, 64-bit prefix sums and input checks
-    uint64_t Pc[L + 1], Px[L + 1];
-    bool neg = dti < 0, big = (dti >> 52) != 0;
-    Pc[0] = 0;
-    Px[0] = 0;
-#pragma unroll
-    for (int r = 1; r <= L; ++r) {
-        const int col = FWD ? r - 1 : L - r;
-        const int64_t cv = active ? stC[lane * K::kStride + col] : 0;
-        const int64_t xv = active ? stX[lane * K::kStride + col] : 0;
-        neg |= (cv < 0) | (xv < 0);
-        big |= ((cv | xv) >> 52) != 0;
-        Pc[r] = Pc[r - 1] + uint64_t(cv);
-        Px[r] = Px[r - 1] + uint64_t(xv);
-    }
-    __syncwarp();  // every lane is done with the staging area before it is reused
-
-    int st = DC_OK;
-    uint64_t bound = 0;
-    if (neg) {
-        st = DC_ERR_NEGATIVE;
-    } else {
-        bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];
-        if (big || bound >= uint64_t(kRangeLimit)) st = DC_ERR_RANGE;
-    }
-    if (!active) return;
-    if (st != DC_OK) {
-        makespan[i] = -int64_t(st);
-        if (nseg) nseg[i] = 0;
-        if (status) status[i] = st;
-#pragma unroll
-        for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
-        return;
-    }
-    if (bound > kNarrowLimit) {  // needs 64-bit values: hand over to the group kernel
-        const uint32_t pos = atomicAdd(wide_count, 1u);
-        wide_list[pos] = uint32_t(i);
-        return;
-    }
-
-    // ---- 32-bit DP
-    uint32_t S[L + 1], Rb[L + 1];
+    T S[L + 1], Rb[L + 1];
 #pragma unroll
     for (int m = 0; m <= L; ++m) {
-        S[m] = uint32_t(FWD ? Pc[m] : Px[m]);
-        Rb[m] = uint32_t(FWD ? Px[m] : Pc[m]);
-    }
-    const uint32_t dtv = uint32_t(dti);
-    const uint32_t c = FWD ? 0u : dtv;
-    uint32_t *lw = region + lane;
-#pragma unroll
-    for (int m = 0; m <= L; ++m) {
+        S[m] = T(FWD ? Pc[m] : Px[m]);
+        Rb[m] = T(FWD ? Px[m] : Pc[m]);
         lw[32 * (K::kOffS + m)] = S[m];
         lw[32 * (K::kOffR + m)] = Rb[m];
     }
-    uint32_t T;
+    const T dtv = T(dti);
+    const T c = FWD ? T(0) : dtv;
+    T Tbest;
     int s;
-    fill32<L, FWD>(S, Rb, dtv, c, lw, T, s);
+    fill<L, FWD, T>(S, Rb, dtv, c, lw, Tbest, s);
 
-    // ---- traceback (Algorithm 3 / 4): from (L, s) step to the lowest k whose
-    // candidate equals the cell value, set p_k / g_k, continue at (k, n-1).
+    // traceback: from (L, s) step to the lowest k whose candidate equals the
+    // cell, set p_k / g_k, continue at (k, n-1)
     uint32_t word = 0;
     int err = 0;
     int m = L, n = s;
+    T cell = Tbest;
     while (n > 1) {
-        const uint32_t R = FWD ? uint32_t(n) * dtv + lw[32 * (K::kOffR + m)]
-                               : lw[32 * (K::kOffR + m)];
-        const uint32_t target =
-            lw[32 * cell_of(L, m, n)] - lw[32 * (K::kOffS + m)] - c;
-        const int colbase = cell_of(L, n - 1, n - 1);  // row n-1 of column n-1
+        const T rm = lds(lw, K::kOffR + m);
+        const T R = FWD ? T(T(n) * dtv + rm) : rm;
+        const T target = T(cell - lds(lw, K::kOffS + m) - c);
         int k = n - 1;
+        T fk = T(0);
         for (; k < m; ++k) {
-            const uint32_t cand =
-                dmax(lw[32 * (colbase + k - (n - 1))], R) - lw[32 * (K::kOffS + k)];
-            if (cand == target) break;
+            fk = prev_cell<L, FWD, T>(lw, k, n - 1, dtv, c);
+            if (T(dmax(fk, R) - lds(lw, K::kOffS + k)) == target) break;
         }
         if (k >= m) {  // cannot happen: the fill and this check use the same arithmetic
             err = 1;
@@ -200,29 +148,208 @@ __global__ void __launch_bounds__(Small<L>::kThreads)
         word |= 1u << ((k - 1) & 31);
         m = k;
         n -= 1;
+        cell = fk;
     }
-    makespan[i] = int64_t(T);
+    makespan[i] = int64_t(Tbest);
     if (nseg) nseg[i] = s;
     if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
     if (W > 0) bits[i * W] = word;
 }
 
+__device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
+{
+    const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
+
+// Issue the copies of tile `base` (rows base..base+rows-1) into the staging area.
 template <int L>
-cudaError_t launch_one(bool forward, int64_t batch, const int64_t *comp, const int64_t *xfer,
+__device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int64_t *comp,
+                                           const int64_t *xfer, int64_t base, int rows, int lane)
+{
+    constexpr int kStride = Small<L, uint32_t>::kStride;
+    const int64_t *gC = comp + base * L;
+    const int64_t *gX = xfer + base * L;
+    const int nel = rows * L;
+    for (int e = lane; e < nel; e += 32) {
+        const int r = e / L, cidx = e - r * L;
+        cp_async8(stC + r * kStride + cidx, gC + e);
+        cp_async8(stX + r * kStride + cidx, gX + e);
+    }
+    cp_async_commit();
+}
+
+// Read this lane's row (processing order) into 64-bit prefix sums; flag bad input.
+template <int L, bool FWD, typename Src>
+__device__ __forceinline__ void row_prefix(Src get, uint64_t (&Pc)[L + 1], uint64_t (&Px)[L + 1],
+                                           bool &neg, bool &big)
+{
+    Pc[0] = 0;
+    Px[0] = 0;
+#pragma unroll
+    for (int r = 1; r <= L; ++r) {
+        const int col = FWD ? r - 1 : L - r;
+        int64_t cv, xv;
+        get(col, cv, xv);
+        neg |= (cv < 0) | (xv < 0);
+        big |= ((cv | xv) >> 52) != 0;
+        Pc[r] = Pc[r - 1] + uint64_t(cv);
+        Px[r] = Px[r - 1] + uint64_t(xv);
+    }
+}
+
+__device__ __forceinline__ void write_failure(int st, int64_t i, int W, int64_t *makespan,
+                                              uint32_t *bits, int32_t *nseg, int32_t *status)
+{
+    makespan[i] = -int64_t(st);
+    if (nseg) nseg[i] = 0;
+    if (status) status[i] = st;
+    for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
+}
+
+// 32-bit pass over the whole batch; persistent warps, cp.async-prefetched tiles.
+template <int L, bool FWD>
+__global__ void __launch_bounds__(32)
+    small_dense_kernel(int64_t batch, const int64_t *__restrict__ comp,
+                       const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
+                       int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,
+                       int32_t *__restrict__ nseg, int32_t *__restrict__ status,
+                       uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list)
+{
+    using K = Small<L, uint32_t>;
+    constexpr int W = (L - 1 + 31) / 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x;
+    int64_t *stC = reinterpret_cast<int64_t *>(smem);
+    int64_t *stX = stC + 32 * K::kStride;
+    uint32_t *lw = reinterpret_cast<uint32_t *>(smem + K::kStageBytes) + lane;
+
+    const int64_t tiles = (batch + 31) / 32;
+    int64_t tile = blockIdx.x;
+    if (tile >= tiles) return;
+    auto rows_of = [&](int64_t t) { return int(batch - t * 32 < 32 ? batch - t * 32 : 32); };
+    stage_tile<L>(stC, stX, comp, xfer, tile * 32, rows_of(tile), lane);
+    for (; tile < tiles; tile += gridDim.x) {
+        const int64_t base = tile * 32;
+        const int rows = rows_of(tile);
+        const int64_t i = base + lane;
+        const bool active = lane < rows;
+        const int64_t dti = active ? __ldg(dt + i) : 0;
+        cp_async_wait_all();
+        __syncwarp();
+        uint64_t Pc[L + 1], Px[L + 1];
+        bool neg = dti < 0, big = (dti >> 52) != 0;
+        row_prefix<L, FWD>(
+            [&](int col, int64_t &cv, int64_t &xv) {
+                cv = active ? stC[lane * K::kStride + col] : 0;
+                xv = active ? stX[lane * K::kStride + col] : 0;
+            },
+            Pc, Px, neg, big);
+        __syncwarp();  // staging free: prefetch the next tile under this tile's DP
+        const int64_t next = tile + gridDim.x;
+        if (next < tiles) stage_tile<L>(stC, stX, comp, xfer, next * 32, rows_of(next), lane);
+        if (!active) continue;
+        int st = DC_OK;
+        uint64_t bound = 0;
+        if (neg) {
+            st = DC_ERR_NEGATIVE;
+        } else {
+            bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];
+            if (big || bound >= uint64_t(kRangeLimit)) st = DC_ERR_RANGE;
+        }
+        if (st != DC_OK) {
+            write_failure(st, i, W, makespan, bits, nseg, status);
+        } else if (bound > kNarrowLimit) {  // needs 64-bit values: work list
+            wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
+        } else {
+            solve<L, FWD, uint32_t>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
+        }
+    }
+    cp_async_wait_all();
+}
+
+// 64-bit pass over the work list (instances whose bound is >= 2^32 - 1).
+template <int L, bool FWD>
+__global__ void __launch_bounds__(32)
+    small_list_kernel(const int64_t *__restrict__ comp, const int64_t *__restrict__ xfer,
+                      const int64_t *__restrict__ dt, int64_t *__restrict__ makespan,
+                      uint32_t *__restrict__ bits, int32_t *__restrict__ nseg,
+                      int32_t *__restrict__ status, const uint32_t *__restrict__ wide_count,
+                      const uint32_t *__restrict__ wide_list)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x;
+    uint64_t *lw = reinterpret_cast<uint64_t *>(smem) + lane;
+    const int64_t count = int64_t(*wide_count);
+    for (int64_t j = int64_t(blockIdx.x) * 32 + lane; j - lane < count; j += int64_t(gridDim.x) * 32) {
+        if (j >= count) continue;
+        const int64_t i = int64_t(wide_list[j]);
+        const int64_t *crow = comp + i * L;
+        const int64_t *xrow = xfer + i * L;
+        const int64_t dti = __ldg(dt + i);
+        uint64_t Pc[L + 1], Px[L + 1];
+        bool neg = false, big = false;  // checked by the dense pass
+        row_prefix<L, FWD>(
+            [&](int col, int64_t &cv, int64_t &xv) {
+                cv = __ldg(crow + col);
+                xv = __ldg(xrow + col);
+            },
+            Pc, Px, neg, big);
+        solve<L, FWD, uint64_t>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
+    }
+}
+
+int g_sm_count = 0;
+
+int sm_count()
+{
+    if (g_sm_count == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_sm_count, cudaDevAttrMultiProcessorCount, dev);
+        if (g_sm_count <= 0) g_sm_count = 152;
+    }
+    return g_sm_count;
+}
+
+template <int L, bool FWD>
+cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
                        const int64_t *dt, int64_t *makespan, uint32_t *bits, int32_t *nseg,
                        int32_t *status, uint32_t *wide_count, uint32_t *wide_list,
                        cudaStream_t stream)
 {
-    using K = Small<L>;
-    const int64_t per_block = int64_t(K::kThreads);
-    const int64_t blocks = (batch + per_block - 1) / per_block;
-    if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
-    if (forward)
-        small_kernel<L, true><<<unsigned(blocks), K::kThreads, K::kSmemBytes, stream>>>(
-            batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
-    else
-        small_kernel<L, false><<<unsigned(blocks), K::kThreads, K::kSmemBytes, stream>>>(
-            batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
+    using K32 = Small<L, uint32_t>;
+    using K64 = Small<L, uint64_t>;
+    static int per_sm = 0;  // resident single-warp CTAs per SM for the dense kernel
+    if (per_sm == 0) {
+        cudaError_t e = cudaFuncSetAttribute(small_dense_kernel<L, FWD>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             K32::kWarpBytes);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(small_list_kernel<L, FWD>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, K64::kTableBytes);
+        if (e != cudaSuccess) return e;
+        int n = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, small_dense_kernel<L, FWD>, 32,
+                                                          K32::kWarpBytes);
+        if (e != cudaSuccess) return e;
+        per_sm = n > 0 ? n : 1;
+    }
+    const int64_t tiles = (batch + 31) / 32;
+    int64_t grid = int64_t(sm_count()) * per_sm;
+    if (grid > tiles) grid = tiles;
+    small_dense_kernel<L, FWD><<<unsigned(grid), 32, K32::kWarpBytes, stream>>>(
+        batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // the list length is known on the device only: size the grid for the worst
+    // case and let surplus warps exit at once
+    int64_t lgrid = (batch + 31) / 32;
+    if (lgrid > int64_t(sm_count()) * 8) lgrid = int64_t(sm_count()) * 8;
+    small_list_kernel<L, FWD><<<unsigned(lgrid), 32, K64::kTableBytes, stream>>>(
+        comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
     return cudaGetLastError();
 }
 
@@ -233,10 +360,12 @@ cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp
                          uint32_t *bits, int32_t *nseg, int32_t *status,
                          uint32_t *wide_count, uint32_t *wide_list, cudaStream_t stream)
 {
-#define DC_SMALL_CASE(LL)                                                                    \
-    case LL:                                                                                 \
-        return launch_one<LL>(forward, batch, comp, xfer, dt, makespan, bits, nseg, status, \
-                              wide_count, wide_list, stream);
+#define DC_SMALL_CASE(LL)                                                                     \
+    case LL:                                                                                  \
+        return forward ? launch_dir<LL, true>(batch, comp, xfer, dt, makespan, bits, nseg,   \
+                                              status, wide_count, wide_list, stream)         \
+                       : launch_dir<LL, false>(batch, comp, xfer, dt, makespan, bits, nseg,  \
+                                               status, wide_count, wide_list, stream);
     switch (L) {
         DC_SMALL_CASE(1) DC_SMALL_CASE(2) DC_SMALL_CASE(3) DC_SMALL_CASE(4)
         DC_SMALL_CASE(5) DC_SMALL_CASE(6) DC_SMALL_CASE(7) DC_SMALL_CASE(8)

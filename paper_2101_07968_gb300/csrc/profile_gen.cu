@@ -1,12 +1,11 @@
 // Seeded synthetic profile generator (stand-in for the real-time profiler of
 // Sec. IV-A, which derives pt, fc, bc, gt and dt from a framework's profiler).
 //
-// One thread per (instance, layer) element; every value is a pure function of
-// (seed, global instance index, field, layer), so any sub-range of a batch can
-// be generated on its own. Integer-only on the device: SplitMix64 draws,
-// multiply-high uniform integers, piecewise-linear log-uniform knots built on the
-// host in double precision, and exact ceiling divisions (float reciprocal
-// estimate + integer remainder correction, no 64-bit divide in the common path).
+// Every value is a pure function of (seed, global instance index, field, layer),
+// so any sub-range of a batch can be generated on its own. Integer-only on the
+// device: SplitMix64 draws, multiply-high uniform integers, piecewise-linear
+// log-uniform knots built on the host in double precision, and exact ceiling
+// divisions by multiply-high with a per-instance reciprocal.
 #include <cmath>
 
 #include "common.cuh"
@@ -55,38 +54,25 @@ __device__ __forceinline__ int64_t loguniform(const int64_t *knots, uint64_t r)
     return t0 + int64_t((uint64_t(t1 - t0) * f) >> 32);
 }
 
-// ceil(a / d), exact, for 0 <= a < 2^62 and 1 <= d < 2^31. Three float
-// estimates of the quotient, each correcting the previous one's remainder,
-// leave |remainder| <= d + 1; two bounded integer steps finish it. The plain
-// 64-bit division is kept only as an unreachable safety net.
-__device__ __forceinline__ uint64_t ceil_div(uint64_t a, uint32_t d)
+// Exact ceil(a / d) for 0 <= a < 2^62 and 1 <= d < 2^31 with m = floor((2^64-1)/d)
+// precomputed once per divisor: q = mulhi(a, m) is floor(a/d) or one less,
+// because a*m/2^64 >= a/d - a*(1 + ((2^64-1) mod d))/(d*2^64) > a/d - 1/4; one
+// remainder step makes it exact.
+__device__ __forceinline__ uint64_t ceil_div(uint64_t a, uint64_t d, uint64_t m)
 {
-    const float rd = __frcp_rn(float(d));
-    uint64_t q = __float2ull_rz(__ull2float_rn(a) * rd);
-    int64_t r = int64_t(a - q * uint64_t(d));
-#pragma unroll
-    for (int it = 0; it < 2; ++it) {
-        q = uint64_t(int64_t(q) + __float2ll_rz(__ll2float_rn(r) * rd));
-        r = int64_t(a - q * uint64_t(d));
-    }
-#pragma unroll
-    for (int it = 0; it < 2; ++it) {
-        if (r < 0) {
-            --q;
-            r += d;
-        }
-        if (r >= int64_t(d)) {
-            ++q;
-            r -= d;
-        }
-    }
-    if (r < 0 || r >= int64_t(d)) {
-        q = a / d;
-        r = int64_t(a - q * d);
+    uint64_t q = __umul64hi(a, m);
+    uint64_t r = a - q * d;
+    if (r >= d) {
+        ++q;
+        r -= d;
     }
     return q + (r != 0 ? 1u : 0u);
 }
 
+// Block-level tiles: a tile is `per` consecutive instances (per = max(1, 256/L)).
+// Phase 1: one thread per instance draws rate, bandwidth and latency and forms
+// the two division magic numbers. Phase 2: every thread produces one (instance,
+// layer) element of the tile, so the four output rows are written coalesced.
 __global__ void __launch_bounds__(256)
     gen_kernel(const __grid_constant__ GenParams g, int64_t *__restrict__ fc,
                int64_t *__restrict__ pt, int64_t *__restrict__ bc, int64_t *__restrict__ gt,
@@ -94,63 +80,69 @@ __global__ void __launch_bounds__(256)
 {
     __shared__ int64_t s_rate[kKnots + 1], s_bw[kKnots + 1];
     __shared__ int64_t s_l0[kFixedMax], s_l1[kFixedMax];
-    const int L = g.L;
-    const int nl = g.layer_mode == DC_LAYERS_FIXED ? L : (g.layer_mode == DC_LAYERS_LOGUNIFORM ? kKnots + 1 : 0);
-    for (int j = threadIdx.x; j <= kKnots; j += blockDim.x) {
+    __shared__ uint64_t s_inst[256][4];  // rate, magic(rate), bw, magic(bw)
+    const int L = g.L, t = threadIdx.x;
+    const int nl = g.layer_mode == DC_LAYERS_FIXED ? L
+                   : (g.layer_mode == DC_LAYERS_LOGUNIFORM ? kKnots + 1 : 0);
+    for (int j = t; j <= kKnots; j += blockDim.x) {
         s_rate[j] = g.rate_knots[j];
         s_bw[j] = g.bw_knots[j];
     }
-    for (int j = threadIdx.x; j < nl; j += blockDim.x) {
+    for (int j = t; j < nl; j += blockDim.x) {
         s_l0[j] = g.layer0[j];
         s_l1[j] = g.layer1[j];
     }
-    __syncthreads();
-
-    const int64_t total = g.batch * L;
-    const int64_t stride = int64_t(gridDim.x) * blockDim.x;
-    int64_t e = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (e >= total) return;
-    // (i, l) of element e, advanced incrementally by the grid stride
-    int64_t i = e / L;
-    int l = int(e - i * L);
-    const int64_t di = stride / L;
-    const int dl = int(stride - di * L);
-    for (; e < total; e += stride) {
-        const int64_t gi = g.inst0 + i;
-        const uint64_t r_rate = splitmix(g.seed, counter(gi, 0, 0));
-        const uint64_t r_bw = splitmix(g.seed, counter(gi, 1, 0));
-        const int64_t rate = g.rate_dist == DC_DIST_LOGUNIFORM
-                                 ? loguniform(s_rate, r_rate)
-                                 : uniform_int(g.rate_lo, g.rate_hi, r_rate);
-        const int64_t bw = g.bw_dist == DC_DIST_LOGUNIFORM ? loguniform(s_bw, r_bw)
-                                                           : uniform_int(g.bw_lo, g.bw_hi, r_bw);
-        int64_t params, flops;
-        if (g.layer_mode == DC_LAYERS_FIXED) {
-            params = s_l0[l];
-            flops = s_l1[l];
-        } else {
-            const uint64_t rp = splitmix(g.seed, counter(gi, 3, l));
-            const uint64_t rf = splitmix(g.seed, counter(gi, 4, l));
-            if (g.layer_mode == DC_LAYERS_LOGUNIFORM) {
-                params = loguniform(s_l0, rp);
-                flops = loguniform(s_l1, rf);
-            } else {
-                params = uniform_int(g.params_lo, g.params_hi, rp);
-                flops = uniform_int(g.flops_lo, g.flops_hi, rf);
-            }
+    const int per = L >= 256 ? 1 : 256 / L;  // instances per tile
+    const int64_t tiles = (g.batch + per - 1) / per;
+    for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+        const int64_t i0 = tile * per;
+        const int n_inst = int(g.batch - i0 < per ? g.batch - i0 : per);
+        __syncthreads();  // tables copied / previous tile done with s_inst
+        if (t < n_inst) {
+            const int64_t i = i0 + t, gi = g.inst0 + i;
+            const uint64_t r_rate = splitmix(g.seed, counter(gi, 0, 0));
+            const uint64_t r_bw = splitmix(g.seed, counter(gi, 1, 0));
+            const int64_t rate = g.rate_dist == DC_DIST_LOGUNIFORM
+                                     ? loguniform(s_rate, r_rate)
+                                     : uniform_int(g.rate_lo, g.rate_hi, r_rate);
+            const int64_t bw = g.bw_dist == DC_DIST_LOGUNIFORM
+                                   ? loguniform(s_bw, r_bw)
+                                   : uniform_int(g.bw_lo, g.bw_hi, r_bw);
+            s_inst[t][0] = uint64_t(rate);
+            s_inst[t][1] = ~uint64_t(0) / uint64_t(rate);
+            s_inst[t][2] = uint64_t(bw);
+            s_inst[t][3] = ~uint64_t(0) / uint64_t(bw);
+            dt[i] = uniform_int(g.dt_lo, g.dt_hi, splitmix(g.seed, counter(gi, 2, 0)));
         }
-        const uint64_t xfer =
-            ceil_div(uint64_t(g.bits) * 1000u * uint64_t(params), uint32_t(bw));
-        fc[e] = int64_t(ceil_div(uint64_t(flops), uint32_t(rate)));
-        bc[e] = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), uint32_t(rate)));
-        pt[e] = int64_t(xfer);
-        gt[e] = int64_t(xfer);
-        if (l == 0) dt[i] = uniform_int(g.dt_lo, g.dt_hi, splitmix(g.seed, counter(gi, 2, 0)));
-        i += di;
-        l += dl;
-        if (l >= L) {
-            l -= L;
-            ++i;
+        __syncthreads();
+        const int total = n_inst * L;
+        for (int e = t; e < total; e += blockDim.x) {
+            const int il = L >= 256 ? 0 : e / L;
+            const int l = e - il * L;
+            const int64_t gi = g.inst0 + i0 + il;
+            int64_t params, flops;
+            if (g.layer_mode == DC_LAYERS_FIXED) {
+                params = s_l0[l];
+                flops = s_l1[l];
+            } else {
+                const uint64_t rp = splitmix(g.seed, counter(gi, 3, l));
+                const uint64_t rf = splitmix(g.seed, counter(gi, 4, l));
+                if (g.layer_mode == DC_LAYERS_LOGUNIFORM) {
+                    params = loguniform(s_l0, rp);
+                    flops = loguniform(s_l1, rf);
+                } else {
+                    params = uniform_int(g.params_lo, g.params_hi, rp);
+                    flops = uniform_int(g.flops_lo, g.flops_hi, rf);
+                }
+            }
+            const uint64_t rate = s_inst[il][0], mr = s_inst[il][1];
+            const uint64_t bw = s_inst[il][2], mb = s_inst[il][3];
+            const uint64_t xfer = ceil_div(uint64_t(g.bits) * 1000u * uint64_t(params), bw, mb);
+            const int64_t o = i0 * L + e;
+            fc[o] = int64_t(ceil_div(uint64_t(flops), rate, mr));
+            bc[o] = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), rate, mr));
+            pt[o] = int64_t(xfer);
+            gt[o] = int64_t(xfer);
         }
     }
 }
@@ -240,9 +232,9 @@ cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_
         knots(c->params_lo, c->params_hi, g.layer0);
         knots(c->flops_lo, c->flops_hi, g.layer1);
     }
-    const int64_t total = c->batch * c->L;
-    int64_t blocks = (total + 255) / 256;
-    if (blocks > 152 * 32) blocks = 152 * 32;
+    const int per = c->L >= 256 ? 1 : 256 / c->L;
+    int64_t blocks = (c->batch + per - 1) / per;
+    if (blocks > 152 * 16) blocks = 152 * 16;
     gen_kernel<<<unsigned(blocks), 256, 0, stream>>>(g, fc, pt, bc, gt, dt);
     return cudaGetLastError();
 }
