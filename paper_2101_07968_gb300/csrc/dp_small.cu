@@ -17,11 +17,14 @@
 //    traceback recovers Path[m][n] as the lowest k whose candidate equals the
 //    cell, which is the k Algorithm 3/4 keeps with its strict-improvement test.
 //    Column 1 (X[m][1] = R(m,1) + S[m] + c) and column L (one cell, the
-//    makespan) are not stored;
+//    makespan) are not stored. The 32-bit pass stores only columns 2..kKeepCols:
+//    the traceback of an s-segment optimum reads columns 1..s-1 only, and s is
+//    small in practice (2-4 on CNN-shaped profiles); an instance whose s needs a
+//    deeper column is re-solved by the 64-bit pass, which keeps every column;
 //  * 32-bit values whenever the instance bound L*dt + sum(xfer) + sum(comp) is
 //    below 2^32 - 1: every DP value and candidate lies in [0, bound], so the
-//    32-bit fill is exact. Other instances are appended to a work list that a
-//    64-bit instantiation of the same kernel solves afterwards;
+//    32-bit fill is exact. Other instances (and the deep ones above) are
+//    appended to a work list that a 64-bit instantiation solves afterwards;
 //  * persistent warps: each warp walks 32-instance tiles; while it solves one
 //    tile, the next tile's rows stream into a padded shared buffer with
 //    cp.async (coalesced 8-byte copies, odd row stride so that every lane reads
@@ -31,9 +34,19 @@
 namespace dc {
 namespace {
 
-template <int L, typename T>
+constexpr int kKeepCols = 4;  // the 32-bit pass stores columns 2..kKeepCols
+
+// index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
+__host__ __device__ constexpr int cell2(int L, int m, int n)
+{
+    return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
+}
+
+// Stored columns 2..C with C = min(keep, L-1); KEEP = L keeps them all.
+template <int L, typename T, int KEEP>
 struct Small {
-    static constexpr int kCells = L >= 2 ? L * (L + 1) / 2 - L - 1 : 0;  // columns 2..L-1
+    static constexpr int kLast = KEEP < L - 1 ? KEEP : L - 1;  // last stored column
+    static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
     static constexpr int kW = sizeof(T) / 4;                            // words per value
     static constexpr int kOffS = kCells;                                // S[0..L]
     static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
@@ -44,17 +57,11 @@ struct Small {
     static constexpr int kWarpBytes = kStageBytes + kTableBytes;
 };
 
-// index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
-__host__ __device__ constexpr int cell2(int L, int m, int n)
-{
-    return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
-}
-
 template <typename T>
 __device__ __forceinline__ T lds(const T *lane_base, int v) { return lane_base[32 * v]; }
 
 // The fill. lw = this lane's values in shared memory (value v at lw[32*v]).
-template <int L, bool FWD, typename T>
+template <int L, bool FWD, typename T, int KEEP>
 __device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], T dtv, T c,
                                      T *lw, T &best_T, int &best_s)
 {
@@ -81,7 +88,7 @@ __device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], 
                 for (int j = 0; j + w < cnt; j += 2 * w) cand[j] = dmin(cand[j], cand[j + w]);
             }
             col[m] = T(cand[0] + S[m] + c);
-            if (n <= L - 1) lw[32 * cell2(L, m, n)] = col[m];
+            if (n <= Small<L, T, KEEP>::kLast) lw[32 * cell2(L, m, n)] = col[m];
         }
         if (col[L] < best_T) {  // strict: the lowest n wins ties
             best_T = col[L];
@@ -91,10 +98,10 @@ __device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], 
 }
 
 // X[k][n-1] during the traceback: column 1 from S and R, others from the table.
-template <int L, bool FWD, typename T>
+template <int L, bool FWD, typename T, int KEEP>
 __device__ __forceinline__ T prev_cell(const T *lw, int k, int nm1, T dtv, T c)
 {
-    using K = Small<L, T>;
+    using K = Small<L, T, KEEP>;
     if (nm1 == 1) {
         const T r = lds(lw, K::kOffR + k);
         return T((FWD ? T(dtv + r) : r) + lds(lw, K::kOffS + k) + c);
@@ -104,12 +111,14 @@ __device__ __forceinline__ T prev_cell(const T *lw, int k, int nm1, T dtv, T c)
 
 // Solve one instance (row data already reduced to 64-bit prefix sums in
 // processing order) and write its outputs.
-template <int L, bool FWD, typename T>
-__device__ __forceinline__ void solve(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+// Returns false (writing nothing) when the optimum's traceback needs a column the
+// pass did not keep; the caller then lists the instance for the full pass.
+template <int L, bool FWD, typename T, int KEEP>
+__device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
                                       int64_t dti, T *lw, int64_t i, int64_t *makespan,
                                       uint32_t *bits, int32_t *nseg, int32_t *status)
 {
-    using K = Small<L, T>;
+    using K = Small<L, T, KEEP>;
     constexpr int W = (L - 1 + 31) / 32;
     T S[L + 1], Rb[L + 1];
 #pragma unroll
@@ -123,7 +132,8 @@ __device__ __forceinline__ void solve(const uint64_t (&Pc)[L + 1], const uint64_
     const T c = FWD ? T(0) : dtv;
     T Tbest;
     int s;
-    fill<L, FWD, T>(S, Rb, dtv, c, lw, Tbest, s);
+    fill<L, FWD, T, KEEP>(S, Rb, dtv, c, lw, Tbest, s);
+    if (s - 1 > K::kLast && s - 1 >= 2) return false;
 
     // traceback: from (L, s) step to the lowest k whose candidate equals the
     // cell, set p_k / g_k, continue at (k, n-1)
@@ -138,7 +148,7 @@ __device__ __forceinline__ void solve(const uint64_t (&Pc)[L + 1], const uint64_
         int k = n - 1;
         T fk = T(0);
         for (; k < m; ++k) {
-            fk = prev_cell<L, FWD, T>(lw, k, n - 1, dtv, c);
+            fk = prev_cell<L, FWD, T, KEEP>(lw, k, n - 1, dtv, c);
             if (T(dmax(fk, R) - lds(lw, K::kOffS + k)) == target) break;
         }
         if (k >= m) {  // cannot happen: the fill and this check use the same arithmetic
@@ -154,6 +164,7 @@ __device__ __forceinline__ void solve(const uint64_t (&Pc)[L + 1], const uint64_
     if (nseg) nseg[i] = s;
     if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
     if (W > 0) bits[i * W] = word;
+    return true;
 }
 
 __device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
@@ -169,7 +180,7 @@ template <int L>
 __device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int64_t *comp,
                                            const int64_t *xfer, int64_t base, int rows, int lane)
 {
-    constexpr int kStride = Small<L, uint32_t>::kStride;
+    constexpr int kStride = Small<L, uint32_t, L>::kStride;
     const int64_t *gC = comp + base * L;
     const int64_t *gX = xfer + base * L;
     const int nel = rows * L;
@@ -218,7 +229,7 @@ __global__ void __launch_bounds__(32)
                        int32_t *__restrict__ nseg, int32_t *__restrict__ status,
                        uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list)
 {
-    using K = Small<L, uint32_t>;
+    using K = Small<L, uint32_t, kKeepCols>;
     constexpr int W = (L - 1 + 31) / 32;
     extern __shared__ __align__(16) unsigned char smem[];
     const int lane = threadIdx.x;
@@ -261,16 +272,17 @@ __global__ void __launch_bounds__(32)
         }
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
-        } else if (bound > kNarrowLimit) {  // needs 64-bit values: work list
+        } else if (bound > kNarrowLimit ||
+                   !solve<L, FWD, uint32_t, kKeepCols>(Pc, Px, dti, lw, i, makespan, bits, nseg,
+                                                       status)) {
+            // 64-bit values, or a traceback deeper than the kept columns: work list
             wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
-        } else {
-            solve<L, FWD, uint32_t>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
         }
     }
     cp_async_wait_all();
 }
 
-// 64-bit pass over the work list (instances whose bound is >= 2^32 - 1).
+// 64-bit pass over the work list, every column kept.
 template <int L, bool FWD>
 __global__ void __launch_bounds__(32)
     small_list_kernel(const int64_t *__restrict__ comp, const int64_t *__restrict__ xfer,
@@ -297,7 +309,7 @@ __global__ void __launch_bounds__(32)
                 xv = __ldg(xrow + col);
             },
             Pc, Px, neg, big);
-        solve<L, FWD, uint64_t>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
+        solve<L, FWD, uint64_t, L>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
     }
 }
 
@@ -320,8 +332,8 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
                        int32_t *status, uint32_t *wide_count, uint32_t *wide_list,
                        cudaStream_t stream)
 {
-    using K32 = Small<L, uint32_t>;
-    using K64 = Small<L, uint64_t>;
+    using K32 = Small<L, uint32_t, kKeepCols>;
+    using K64 = Small<L, uint64_t, L>;
     static int per_sm = 0;  // resident single-warp CTAs per SM for the dense kernel
     if (per_sm == 0) {
         cudaError_t e = cudaFuncSetAttribute(small_dense_kernel<L, FWD>,

@@ -22,13 +22,9 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
         uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
         cudaError_t e = cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
         if (e != cudaSuccess) return e;
-        e = launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, count,
-                         list, stream);
-        if (e != cudaSuccess) return e;
-        // 64-bit leftovers: a persistent grid that reads the list length on the device
-        const int64_t grid = batch < 1216 ? batch : 1216;
-        return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                            count, list, nullptr, grid, stream);
+        // 32-bit pass over the batch, then a 64-bit pass over the instances it listed
+        return launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                            count, list, stream);
     }
     if (L <= kSmemTableLMax) {
         const int64_t grid = batch < 152 * 32 ? batch : 152 * 32;

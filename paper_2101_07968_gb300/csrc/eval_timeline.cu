@@ -12,8 +12,8 @@
 // Inputs are checked like the solver's (negative -> -3, bound >= 2^52 -> -4).
 //
 // For L <= 32 a warp first copies its 32 instances' rows into shared memory with
-// coalesced loads (odd row stride: conflict-free per-lane row reads); longer
-// rows are read by each thread directly.
+// coalesced asynchronous copies (odd row stride: conflict-free per-lane row
+// reads); longer rows are read by each thread directly.
 #include "common.cuh"
 
 namespace dc {
@@ -88,6 +88,12 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+__device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
+{
+    const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
+
 template <bool FWD>
 __global__ void __launch_bounds__(32 * kEvalWarps)
     eval_staged_kernel(int64_t batch, int L, const int64_t *__restrict__ comp,
@@ -108,11 +114,14 @@ __global__ void __launch_bounds__(32 * kEvalWarps)
         const int64_t *gC = comp + base * L;
         const int64_t *gX = xfer + base * L;
         __syncwarp();
+        // all copies in flight at once (no register round trip), then one wait
         for (int e = lane; e < nel; e += 32) {
             const int r = e / L, cidx = e - r * L;
-            stC[r * stride + cidx] = __ldg(gC + e);
-            stX[r * stride + cidx] = __ldg(gX + e);
+            cp_async8(stC + r * stride + cidx, gC + e);
+            cp_async8(stX + r * stride + cidx, gX + e);
         }
+        asm volatile("cp.async.commit_group;\n" ::: "memory");
+        asm volatile("cp.async.wait_group 0;\n" ::: "memory");
         __syncwarp();
         if (lane >= rows) continue;
         const int64_t i = base + lane;

@@ -69,19 +69,22 @@ __device__ __forceinline__ uint64_t ceil_div(uint64_t a, uint64_t d, uint64_t m)
     return q + (r != 0 ? 1u : 0u);
 }
 
-// Block-level tiles: a tile is `per` consecutive instances (per = max(1, 256/L)).
-// Phase 1: one thread per instance draws rate, bandwidth and latency and forms
-// the two division magic numbers. Phase 2: every thread produces one (instance,
-// layer) element of the tile, so the four output rows are written coalesced.
-__global__ void __launch_bounds__(256)
+// Warp-level tiles of 32 consecutive instances. Phase 1: lane j draws rate,
+// bandwidth and latency of instance j and forms the two division magic numbers
+// (32 instances' 64-bit divisions run side by side). Phase 2: the warp walks the
+// tile's 32*L (instance, layer) elements 32 at a time, so the four output rows
+// are written coalesced. Only __syncwarp between the phases.
+constexpr int kGenWarps = 8;
+
+__global__ void __launch_bounds__(32 * kGenWarps)
     gen_kernel(const __grid_constant__ GenParams g, int64_t *__restrict__ fc,
                int64_t *__restrict__ pt, int64_t *__restrict__ bc, int64_t *__restrict__ gt,
                int64_t *__restrict__ dt)
 {
     __shared__ int64_t s_rate[kKnots + 1], s_bw[kKnots + 1];
     __shared__ int64_t s_l0[kFixedMax], s_l1[kFixedMax];
-    __shared__ uint64_t s_inst[256][4];  // rate, magic(rate), bw, magic(bw)
-    const int L = g.L, t = threadIdx.x;
+    __shared__ uint64_t s_inst[kGenWarps][4][32];  // rate, magic(rate), bw, magic(bw)
+    const int L = g.L, t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nl = g.layer_mode == DC_LAYERS_FIXED ? L
                    : (g.layer_mode == DC_LAYERS_LOGUNIFORM ? kKnots + 1 : 0);
     for (int j = t; j <= kKnots; j += blockDim.x) {
@@ -92,14 +95,17 @@ __global__ void __launch_bounds__(256)
         s_l0[j] = g.layer0[j];
         s_l1[j] = g.layer1[j];
     }
-    const int per = L >= 256 ? 1 : 256 / L;  // instances per tile
-    const int64_t tiles = (g.batch + per - 1) / per;
-    for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-        const int64_t i0 = tile * per;
-        const int n_inst = int(g.batch - i0 < per ? g.batch - i0 : per);
-        __syncthreads();  // tables copied / previous tile done with s_inst
-        if (t < n_inst) {
-            const int64_t i = i0 + t, gi = g.inst0 + i;
+    __syncthreads();
+    uint64_t(*si)[32] = s_inst[warp];
+    const int step_i = 32 / L, step_l = 32 % L;  // advance of (instance, layer) per 32 elements
+    const int64_t tiles = (g.batch + 31) / 32;
+    for (int64_t tile = int64_t(blockIdx.x) * kGenWarps + warp; tile < tiles;
+         tile += int64_t(gridDim.x) * kGenWarps) {
+        const int64_t i0 = tile * 32;
+        const int n_inst = int(g.batch - i0 < 32 ? g.batch - i0 : 32);
+        __syncwarp();  // previous tile done with si
+        if (lane < n_inst) {
+            const int64_t i = i0 + lane, gi = g.inst0 + i;
             const uint64_t r_rate = splitmix(g.seed, counter(gi, 0, 0));
             const uint64_t r_bw = splitmix(g.seed, counter(gi, 1, 0));
             const int64_t rate = g.rate_dist == DC_DIST_LOGUNIFORM
@@ -108,17 +114,16 @@ __global__ void __launch_bounds__(256)
             const int64_t bw = g.bw_dist == DC_DIST_LOGUNIFORM
                                    ? loguniform(s_bw, r_bw)
                                    : uniform_int(g.bw_lo, g.bw_hi, r_bw);
-            s_inst[t][0] = uint64_t(rate);
-            s_inst[t][1] = ~uint64_t(0) / uint64_t(rate);
-            s_inst[t][2] = uint64_t(bw);
-            s_inst[t][3] = ~uint64_t(0) / uint64_t(bw);
+            si[0][lane] = uint64_t(rate);
+            si[1][lane] = ~uint64_t(0) / uint64_t(rate);
+            si[2][lane] = uint64_t(bw);
+            si[3][lane] = ~uint64_t(0) / uint64_t(bw);
             dt[i] = uniform_int(g.dt_lo, g.dt_hi, splitmix(g.seed, counter(gi, 2, 0)));
         }
-        __syncthreads();
+        __syncwarp();
         const int total = n_inst * L;
-        for (int e = t; e < total; e += blockDim.x) {
-            const int il = L >= 256 ? 0 : e / L;
-            const int l = e - il * L;
+        int il = lane / L, l = lane - (lane / L) * L;
+        for (int e = lane; e < total; e += 32) {
             const int64_t gi = g.inst0 + i0 + il;
             int64_t params, flops;
             if (g.layer_mode == DC_LAYERS_FIXED) {
@@ -135,14 +140,20 @@ __global__ void __launch_bounds__(256)
                     flops = uniform_int(g.flops_lo, g.flops_hi, rf);
                 }
             }
-            const uint64_t rate = s_inst[il][0], mr = s_inst[il][1];
-            const uint64_t bw = s_inst[il][2], mb = s_inst[il][3];
+            const uint64_t rate = si[0][il], mr = si[1][il];
+            const uint64_t bw = si[2][il], mb = si[3][il];
             const uint64_t xfer = ceil_div(uint64_t(g.bits) * 1000u * uint64_t(params), bw, mb);
             const int64_t o = i0 * L + e;
             fc[o] = int64_t(ceil_div(uint64_t(flops), rate, mr));
             bc[o] = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), rate, mr));
             pt[o] = int64_t(xfer);
             gt[o] = int64_t(xfer);
+            il += step_i;
+            l += step_l;
+            if (l >= L) {
+                l -= L;
+                ++il;
+            }
         }
     }
 }
@@ -232,10 +243,10 @@ cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_
         knots(c->params_lo, c->params_hi, g.layer0);
         knots(c->flops_lo, c->flops_hi, g.layer1);
     }
-    const int per = c->L >= 256 ? 1 : 256 / c->L;
-    int64_t blocks = (c->batch + per - 1) / per;
-    if (blocks > 152 * 16) blocks = 152 * 16;
-    gen_kernel<<<unsigned(blocks), 256, 0, stream>>>(g, fc, pt, bc, gt, dt);
+    const int64_t tiles = (c->batch + 31) / 32;
+    int64_t blocks = (tiles + kGenWarps - 1) / kGenWarps;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    gen_kernel<<<unsigned(blocks), 32 * kGenWarps, 0, stream>>>(g, fc, pt, bc, gt, dt);
     return cudaGetLastError();
 }
 
