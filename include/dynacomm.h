@@ -162,6 +162,35 @@ dc_status dc_eval_timeline_batch(int64_t batch, int32_t L, int32_t dir, const in
                                  const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                                  int64_t *makespan, cudaStream_t stream);
 
+/* ------------------------------------------------------------------------
+ * dc_schedule_batch_static -- the paper has no counterpart: this is a
+ * deployment variant of the two schedule calls above for callers that cannot
+ * allocate device memory where they schedule (a scheduler embedded in a
+ * training runtime whose allocator owns all device memory and refuses other
+ * allocations once training runs, or one that schedules inside the idle window
+ * between a gradient push and the next pull, where a cudaMalloc that can
+ * synchronise the device is not acceptable). It takes no workspace.
+ *
+ * dir 0 solves Algorithm 3 (comp = fc, xfer = pt), dir 1 Algorithm 4
+ * (comp = bc, xfer = gt); inputs, outputs and per-instance status are exactly
+ * those of dc_schedule_forward_batch / dc_schedule_backward_batch.
+ * Limits: 1 <= L <= 16 (else DC_ERR_BAD_SHAPE); batch <= 1,048,576
+ * (DC_STATIC_MAX_BATCH; a larger batch returns DC_ERR_WORKSPACE, launching
+ * nothing).
+ * Scratch: a 4 MiB + 256 B array in the library's device memory, held by every
+ * GPU that loads the library until the process exits, shared by all calls on a
+ * device: calls that overlap on one GPU race on it, so serialise them (one
+ * stream, or an event between them). Each call clears what must start at zero.
+ * The first call on a device looks up the array's device address (a
+ * cudaGetSymbolAddress with that device current); make that first call before
+ * any stream capture. No cudaMalloc, cudaFree or other allocating call is made.
+ * ---------------------------------------------------------------------- */
+#define DC_STATIC_MAX_BATCH 1048576
+dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,
+                                   const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                                   uint32_t *bits, int32_t *nseg, int32_t *status,
+                                   cudaStream_t stream);
+
 /* Static description of a status code. Never NULL. */
 const char *dc_status_string(dc_status s);
 

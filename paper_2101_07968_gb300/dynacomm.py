@@ -22,6 +22,7 @@ LIB_PATH = os.path.join(_PKG, "libdynacomm.so")
 DC_OK, DC_ERR_NULL, DC_ERR_BAD_SHAPE, DC_ERR_NEGATIVE, DC_ERR_RANGE = 0, 1, 2, 3, 4
 DC_ERR_WORKSPACE, DC_ERR_CUDA, DC_ERR_BAD_CONFIG, DC_ERR_INTERNAL = 5, 6, 7, 8
 DC_L_MAX = 4096
+DC_STATIC_MAX_BATCH = 1048576
 FWD, BWD = 0, 1
 
 
@@ -59,6 +60,8 @@ _SIGNATURES = {
     "dc_schedule_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
                                           _SZ, _VP]),
     "dc_eval_timeline_batch": (_I32, [_I64, _I32, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
+    "dc_schedule_batch_static": (_I32, [_I32, _I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                        _VP]),
     "dc_status_string": (ctypes.c_char_p, [_I32]),
     "dc_roof_int_probe": (_I32, [_I32, _I32, _I32, _I64, _VP, _VP]),
 }
@@ -168,6 +171,16 @@ def dc_schedule_backward_batch(batch, L, bc, gt, dt, makespan, bits, nseg, statu
     return int(lib().dc_schedule_backward_batch(
         int(batch), int(L), _ptr(bc), _ptr(gt), _ptr(dt), _ptr(makespan), _ptr(bits),
         _ptr(nseg), _ptr(status), _ptr(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def dc_schedule_batch_static(direction, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                             stream=None) -> int:
+    """Workspace-free solve for 1 <= L <= 16 and batch <= DC_STATIC_MAX_BATCH, for
+    callers that cannot allocate device memory; its scratch is a fixed array in the
+    library shared by every call on a device (overlapping calls race)."""
+    return int(lib().dc_schedule_batch_static(
+        int(direction), int(batch), int(L), _ptr(comp), _ptr(xfer), _ptr(dt), _ptr(makespan),
+        _ptr(bits), _ptr(nseg), _ptr(status), _stream(stream)))
 
 
 def dc_eval_timeline_batch(batch, L, direction, comp, xfer, dt, bits, makespan,
