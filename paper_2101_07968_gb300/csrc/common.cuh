@@ -10,8 +10,10 @@
 
 namespace dc {
 
-constexpr int kSmallLMax = 16;       // thread-per-instance kernel covers 1 <= L <= 16
+constexpr int kSmallLMax = 16;       // unrolled thread-per-instance kernel: 1 <= L <= 16
+constexpr int kMidLMax = 64;         // looped thread-per-instance kernel: 17 <= L <= 64
 constexpr int kSmemTableLMax = 64;   // group kernel keeps its DP table on chip up to here
+constexpr int64_t kMidSlots = 152 * 16 * 32;  // traceback slots of the looped kernel
 constexpr int64_t kRangeLimit = int64_t(1) << 52;
 constexpr uint64_t kNarrowLimit = 0xFFFFFFFEull;  // bound that lets a DP run in 32 bits
 
@@ -37,12 +39,15 @@ inline int64_t table_slots(int L)
     return s;
 }
 
+size_t mid_scratch_bytes(int L);  // dp_mid.cu
+
 struct Workspace {
-    // Layout: [0, 256) header (wide-list counter), [256, 256 + 4*batch) wide list
-    // (only when L <= kSmallLMax), then 256-aligned per-slot DP tables (L > 64).
+    // Layout: [0, 256) header (work-list counter, tile ticket), [256, 256 + 4*batch)
+    // work list (L <= kMidLMax), then, 256-aligned, the looped kernel's traceback
+    // slots (17 <= L <= 64) or the per-CTA DP tables of the group kernel (L > 64).
     static size_t list_bytes(int64_t batch, int L)
     {
-        return L <= kSmallLMax ? size_t(batch) * 4 : 0;
+        return L <= kMidLMax ? size_t(batch) * 4 : 0;
     }
     static size_t table_offset(int64_t batch, int L)
     {
@@ -56,6 +61,7 @@ struct Workspace {
     }
     static size_t bytes(int64_t batch, int L)
     {
+        if (L > kSmallLMax && L <= kMidLMax) return table_offset(batch, L) + mid_scratch_bytes(L);
         return table_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
     }
 };
@@ -89,6 +95,10 @@ cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp
                          uint32_t *bits, int32_t *nseg, int32_t *status,
                          const uint32_t *list_count, const uint32_t *list, void *tables,
                          int64_t grid, cudaStream_t stream);
+cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
+                       const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                       uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
+                       uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream);
 cudaError_t launch_eval(bool forward, int64_t batch, int L, const int64_t *comp,
                         const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                         int64_t *makespan, cudaStream_t stream);

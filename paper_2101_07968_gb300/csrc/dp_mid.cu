@@ -1,0 +1,233 @@
+// Thread-per-instance DynaComm DP for 17 <= L <= 64 (Eq. 8 / Algorithm 3 and
+// Eq. 9 / Algorithm 4), 32-bit arithmetic, runtime loops.
+//
+// Same processing-order template as the other kernels:
+//   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
+//
+// Design (GB300):
+//  * one instance per thread; the lane's S, R and current column live in its
+//    slice of shared memory (lane-interleaved: value v at word 32*v + lane, so a
+//    warp's accesses never conflict);
+//  * register blocking: a column is filled in blocks of kB = 8 consecutive rows
+//    held in registers; every X[k][n-1], S[k] pair read from shared memory feeds
+//    kB transitions (max, subtract, min). Rows are visited top-down so that the
+//    column is updated in place: a block reads only rows below its own top,
+//    which still hold column n-1;
+//  * value-only fill with deferred argmin, as in the short-L kernel: columns
+//    2..kKeep are written to a per-thread slot of the caller's workspace (L2
+//    resident, coalesced across the warp) and the traceback re-derives each
+//    Path[m][n] as the lowest k whose candidate equals the cell. Instances whose
+//    optimum needs a deeper column, or whose values need 64 bits, are put on a
+//    work list that the CTA-per-instance kernel solves afterwards;
+//  * persistent single-warp CTAs claim 32-instance tiles from an atomic ticket,
+//    so the long, uneven per-tile work balances across the GPU.
+#include "common.cuh"
+
+namespace dc {
+namespace {
+
+constexpr int kB = 8;      // rows per register block
+constexpr int kKeep = 8;  // last column kept for the traceback
+
+__host__ __device__ inline int mid_keep_last(int L) { return L - 1 < kKeep ? L - 1 : kKeep; }
+// stored cell (m, n), 2 <= n <= keep_last
+__host__ __device__ inline int mid_cell(int L, int m, int n)
+{
+    return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
+}
+__host__ __device__ inline int mid_cells(int L)
+{
+    const int c = mid_keep_last(L);
+    return c >= 2 ? mid_cell(L, L, c) + 1 : 0;
+}
+
+template <bool FWD>
+__global__ void __launch_bounds__(32)
+    mid_kernel(int64_t batch, int L, const int64_t *__restrict__ comp,
+               const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
+               int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,
+               int32_t *__restrict__ nseg, int32_t *__restrict__ status,
+               uint32_t *__restrict__ ticket, uint32_t *__restrict__ list_count,
+               uint32_t *__restrict__ list, uint32_t *__restrict__ tb, int64_t nslots)
+{
+    extern __shared__ uint32_t smem[];
+    const int lane = threadIdx.x;
+    const int W = words_for(L);
+    uint32_t *lw = smem + lane;  // S at v in [0, L], R at [L+1, 2L+1], col at [2L+2, 3L+2]
+    const int oR = L + 1, oC = 2 * (L + 1);
+    const int64_t slot = int64_t(blockIdx.x) * 32 + lane;
+    uint32_t *myslot = tb + slot;  // cell c at myslot[c * nslots]
+    const int keep = mid_keep_last(L);
+    const int64_t tiles = (batch + 31) / 32;
+
+    for (;;) {
+        uint32_t tile = 0;
+        if (lane == 0) tile = atomicAdd(ticket, 1u);
+        tile = __shfl_sync(0xffffffffu, tile, 0);
+        if (int64_t(tile) >= tiles) break;
+        const int64_t i = int64_t(tile) * 32 + lane;
+        if (i >= batch) continue;
+
+        // ---- row -> 32-bit prefix sums in processing order, input checks
+        const int64_t *crow = comp + i * L, *xrow = xfer + i * L;
+        const int64_t dti = __ldg(dt + i);
+        bool neg = dti < 0, big = (dti >> 52) != 0;
+        uint64_t pc = 0, px = 0;
+        lw[0] = 0u;
+        lw[32 * oR] = 0u;
+        for (int r = 1; r <= L; ++r) {
+            const int col = FWD ? r - 1 : L - r;
+            const int64_t cv = __ldg(crow + col), xv = __ldg(xrow + col);
+            neg |= (cv < 0) | (xv < 0);
+            big |= ((cv | xv) >> 52) != 0;
+            pc += uint64_t(cv);
+            px += uint64_t(xv);
+            lw[32 * r] = uint32_t(FWD ? pc : px);         // S
+            lw[32 * (oR + r)] = uint32_t(FWD ? px : pc);  // R base
+        }
+        if (neg || big || exceeds_range(L, dti, pc, px)) {
+            const int st = neg ? DC_ERR_NEGATIVE : DC_ERR_RANGE;
+            makespan[i] = -int64_t(st);
+            if (nseg) nseg[i] = 0;
+            if (status) status[i] = st;
+            for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
+            continue;
+        }
+        if (pc + px + uint64_t(L) * uint64_t(dti) > kNarrowLimit) {
+            list[atomicAdd(list_count, 1u)] = uint32_t(i);
+            continue;
+        }
+
+        // ---- fill
+        const uint32_t dtv = uint32_t(dti);
+        const uint32_t c = FWD ? 0u : dtv;
+        for (int m = 1; m <= L; ++m) {
+            const uint32_t rb = lw[32 * (oR + m)];
+            lw[32 * (oC + m)] = (FWD ? dtv + rb : rb) + lw[32 * m] + c;
+        }
+        uint32_t Tbest = lw[32 * (oC + L)];
+        int s = 1;
+        for (int n = 2; n <= L; ++n) {
+            const uint32_t ndt = uint32_t(n) * dtv;
+            for (int top = L; top >= n; top -= kB) {
+                const int bot = top - kB + 1 > n ? top - kB + 1 : n;
+                uint32_t R[kB], best[kB];
+#pragma unroll
+                for (int j = 0; j < kB; ++j) {
+                    const int m = bot + j <= top ? bot + j : top;
+                    const uint32_t rb = lw[32 * (oR + m)];
+                    R[j] = FWD ? ndt + rb : rb;
+                    best[j] = 0xffffffffu;
+                }
+                // k below the block: every row of the block takes it
+                for (int k = n - 1; k < bot; ++k) {
+                    const uint32_t v = lw[32 * (oC + k)], sk = lw[32 * k];
+#pragma unroll
+                    for (int j = 0; j < kB; ++j) best[j] = dmin(best[j], dmax(v, R[j]) - sk);
+                }
+                // k inside the block: row bot+j takes k < bot+j
+#pragma unroll
+                for (int t = 0; t < kB - 1; ++t) {
+                    const int k = bot + t;
+                    if (k >= top) break;
+                    const uint32_t v = lw[32 * (oC + k)], sk = lw[32 * k];
+#pragma unroll
+                    for (int j = t + 1; j < kB; ++j) best[j] = dmin(best[j], dmax(v, R[j]) - sk);
+                }
+#pragma unroll
+                for (int j = 0; j < kB; ++j) {
+                    const int m = bot + j;
+                    if (m <= top) {
+                        const uint32_t val = best[j] + lw[32 * m] + c;
+                        lw[32 * (oC + m)] = val;
+                        if (n <= keep) myslot[int64_t(mid_cell(L, m, n)) * nslots] = val;
+                    }
+                }
+            }
+            const uint32_t last = lw[32 * (oC + L)];
+            if (last < Tbest) {  // strict: the lowest n wins ties
+                Tbest = last;
+                s = n;
+            }
+        }
+        if (s - 1 > keep && s - 1 >= 2) {  // traceback would need an unkept column
+            list[atomicAdd(list_count, 1u)] = uint32_t(i);
+            continue;
+        }
+
+        // ---- traceback: lowest k whose candidate equals the cell
+        uint32_t word0 = 0u, word1 = 0u;  // L <= 64: W <= 2
+        int err = 0, m = L, n = s;
+        uint32_t cell = Tbest;
+        while (n > 1) {
+            const uint32_t rm = lw[32 * (oR + m)];
+            const uint32_t R = FWD ? uint32_t(n) * dtv + rm : rm;
+            const uint32_t target = cell - lw[32 * m] - c;
+            int k = n - 1;
+            uint32_t fk = 0;
+            for (; k < m; ++k) {
+                if (n - 1 == 1) {
+                    const uint32_t rb = lw[32 * (oR + k)];
+                    fk = (FWD ? dtv + rb : rb) + lw[32 * k] + c;
+                } else {
+                    fk = myslot[int64_t(mid_cell(L, k, n - 1)) * nslots];
+                }
+                if (dmax(fk, R) - lw[32 * k] == target) break;
+            }
+            if (k >= m) {
+                err = 1;
+                break;
+            }
+            if (k - 1 < 32)
+                word0 |= 1u << (k - 1);
+            else
+                word1 |= 1u << (k - 33);
+            m = k;
+            n -= 1;
+            cell = fk;
+        }
+        makespan[i] = int64_t(Tbest);
+        if (nseg) nseg[i] = s;
+        if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+        bits[i * W] = word0;
+        if (W > 1) bits[i * W + 1] = word1;
+    }
+}
+
+}  // namespace
+
+size_t mid_scratch_bytes(int L) { return size_t(kMidSlots) * size_t(mid_cells(L)) * 4; }
+
+cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
+                       const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                       uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
+                       uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream)
+{
+    const size_t smem = size_t(3) * (L + 1) * 32 * 4;
+    static bool attr = false;
+    if (!attr) {
+        const int most = 3 * (kMidLMax + 1) * 32 * 4;
+        cudaError_t e = cudaFuncSetAttribute(mid_kernel<true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(mid_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     most);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    int64_t grid = kMidSlots / 32;
+    const int64_t tiles = (batch + 31) / 32;
+    if (grid > tiles) grid = tiles;
+    if (forward)
+        mid_kernel<true><<<unsigned(grid), 32, smem, stream>>>(batch, L, comp, xfer, dt, makespan,
+                                                             bits, nseg, status, ticket,
+                                                             list_count, list, tb, kMidSlots);
+    else
+        mid_kernel<false><<<unsigned(grid), 32, smem, stream>>>(batch, L, comp, xfer, dt,
+                                                              makespan, bits, nseg, status,
+                                                              ticket, list_count, list, tb,
+                                                              kMidSlots);
+    return cudaGetLastError();
+}
+
+}  // namespace dc

@@ -34,7 +34,16 @@
 namespace dc {
 namespace {
 
-constexpr int kKeepCols = 4;  // the 32-bit pass stores columns 2..kKeepCols
+#ifndef DC_KEEP_COLS
+#define DC_KEEP_COLS 4
+#endif
+#ifndef DC_SMALL_MINB
+#define DC_SMALL_MINB 1
+#endif
+#ifndef DC_TREE_MIN
+#define DC_TREE_MIN 1
+#endif
+constexpr int kKeepCols = DC_KEEP_COLS;  // the 32-bit pass stores columns 2..kKeepCols
 
 // index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
 __host__ __device__ constexpr int cell2(int L, int m, int n)
@@ -82,10 +91,15 @@ __device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], 
             const int cnt = m - n + 1;  // k = n-1 .. m-1
 #pragma unroll
             for (int j = 0; j < cnt; ++j) cand[j] = T(dmax(col[n - 1 + j], R) - S[n - 1 + j]);
+            if (DC_TREE_MIN) {  // balanced tree: log-depth chains
 #pragma unroll
-            for (int w = 1; w < cnt; w *= 2) {
+                for (int w = 1; w < cnt; w *= 2) {
 #pragma unroll
-                for (int j = 0; j + w < cnt; j += 2 * w) cand[j] = dmin(cand[j], cand[j + w]);
+                    for (int j = 0; j + w < cnt; j += 2 * w) cand[j] = dmin(cand[j], cand[j + w]);
+                }
+            } else {
+#pragma unroll
+                for (int j = 1; j < cnt; ++j) cand[0] = dmin(cand[0], cand[j]);
             }
             col[m] = T(cand[0] + S[m] + c);
             if (n <= Small<L, T, KEEP>::kLast) lw[32 * cell2(L, m, n)] = col[m];
@@ -222,7 +236,7 @@ __device__ __forceinline__ void write_failure(int st, int64_t i, int W, int64_t 
 
 // 32-bit pass over the whole batch; persistent warps, cp.async-prefetched tiles.
 template <int L, bool FWD>
-__global__ void __launch_bounds__(32)
+__global__ void __launch_bounds__(32, DC_SMALL_MINB)
     small_dense_kernel(int64_t batch, const int64_t *__restrict__ comp,
                        const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
                        int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,

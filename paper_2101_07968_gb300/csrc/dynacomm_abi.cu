@@ -26,10 +26,21 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
         return launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
                             count, list, stream);
     }
-    if (L <= kSmemTableLMax) {
-        const int64_t grid = batch < 152 * 32 ? batch : 152 * 32;
+    if (L <= kMidLMax) {
+        // looped 32-bit pass (tile ticket + work list in the header), then the
+        // CTA-per-instance kernel over the listed 64-bit / deep instances
+        uint32_t *count = reinterpret_cast<uint32_t *>(ws);
+        uint32_t *ticket = count + 1;
+        uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
+        uint32_t *tb = reinterpret_cast<uint32_t *>(ws + Workspace::table_offset(batch, L));
+        cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(uint32_t), stream);
+        if (e != cudaSuccess) return e;
+        e = launch_mid(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket,
+                       count, list, tb, stream);
+        if (e != cudaSuccess) return e;
+        const int64_t grid = batch < 152 * 8 ? batch : 152 * 8;
         return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                            nullptr, nullptr, nullptr, grid, stream);
+                            count, list, nullptr, grid, stream);
     }
     const int64_t slots = int64_t(Workspace::slots(batch, L));
     return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,

@@ -47,7 +47,10 @@ def test_workspace_query(lib):
     assert dc.dc_schedule_workspace_bytes(10, 0) == 0
     assert dc.dc_schedule_workspace_bytes(10, 4097) == 0
     assert dc.dc_schedule_workspace_bytes(1000, 16) >= 256 + 4000
-    assert dc.dc_schedule_workspace_bytes(1000, 17) == 256
+    # 17 <= L <= 64: work list plus fixed per-thread traceback slots
+    mid = dc.dc_schedule_workspace_bytes(1000, 54)
+    assert mid >= 256 + 4000 and mid == dc.dc_schedule_workspace_bytes(1000, 54)
+    assert abs(dc.dc_schedule_workspace_bytes(2000, 54) - mid - 4000) < 256
     # long L: one DP-table slot per concurrently solved instance
     one = dc.dc_schedule_workspace_bytes(1, 1024)
     assert one >= 1024 * 1025 // 2 * 8
