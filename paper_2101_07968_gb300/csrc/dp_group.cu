@@ -6,11 +6,12 @@
 //
 // Same processing-order template as the small kernel:
 //   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
-// Column n is filled in parallel (one row m per thread, strided), columns run in
-// sequence with a CTA barrier between them; two column buffers live in shared
-// memory and every finished cell is also written to the instance's DP table
-// (shared memory for L <= 64, otherwise a per-CTA slot of the caller's
-// workspace). After the fill, warp 0 picks the lowest n minimising X[L][n] and
+// Column n's (row block, k chunk) tiles are spread over the CTA's threads (8 rows
+// x up to 64 candidates per tile, register-blocked), partial row minima are
+// combined with shared-memory atomicMin, then the column is finalised; columns
+// run in sequence with CTA barriers between them. Every finished cell is also
+// written to the instance's DP table (shared memory for L <= 64, otherwise a
+// per-CTA slot of the caller's workspace). After the fill, warp 0 picks the lowest n minimising X[L][n] and
 // walks the traceback, finding each Path[m][n] (the lowest k whose candidate
 // equals the cell) with one ballot per 32 candidates.
 #include "common.cuh"
@@ -29,10 +30,14 @@ struct GroupArgs {
     unsigned char *tables;  // nullptr: DP table in shared memory
 };
 
-// Shared-memory layout: four (L+1)-entry arrays sized for 64-bit values
-// (S, R, two column buffers), the decision words, a 256-byte scan scratch, and
-// the DP table when it stays on chip.
-__host__ __device__ inline size_t group_arrays_bytes(int L) { return size_t(4) * (L + 1) * 8; }
+// Shared-memory layout: five arrays of Ls = L + 1 + (L + 1)/32 + 1 entries sized
+// for 64-bit values (S, R, two column buffers, per-row partial minima), indexed
+// through skew(k) = k + k/32 so that tiles whose k ranges start 64 apart hit
+// different banks; then the decision words, a 256-byte scan scratch, and the DP
+// table when it stays on chip.
+__host__ __device__ inline int group_ls(int L) { return L + 1 + (L + 1) / 32 + 1; }
+__device__ __forceinline__ int skew(int k) { return k + (k >> 5); }
+__host__ __device__ inline size_t group_arrays_bytes(int L) { return size_t(5) * group_ls(L) * 8; }
 __host__ __device__ inline size_t group_bits_bytes(int L)
 {
     return (size_t(words_for(L) + 1) * 4 + 15) / 16 * 16;
@@ -59,7 +64,6 @@ __device__ void block_prefix_u64(uint64_t *v, int L, uint64_t *scratch /* >= 16 
         acc += v[j];
         v[j] = acc;
     }
-    // exclusive scan of per-thread totals: warp-level, then across warps
     const int lane = t & 31, warp = t >> 5, nw = (nt + 31) >> 5;
     uint64_t x = acc;
 #pragma unroll
@@ -83,52 +87,110 @@ __device__ void block_prefix_u64(uint64_t *v, int L, uint64_t *scratch /* >= 16 
     __syncthreads();
 }
 
+__device__ __forceinline__ void atomic_min_T(uint32_t *p, uint32_t v) { atomicMin(p, v); }
+__device__ __forceinline__ void atomic_min_T(uint64_t *p, uint64_t v)
+{
+    atomicMin(reinterpret_cast<unsigned long long *>(p), static_cast<unsigned long long>(v));
+}
+
+constexpr int kRB = 8;   // rows per tile
+constexpr int kKC = 64;  // k per tile
+
+// Column n's work is the set of (row block b, k chunk j) tiles: block b holds
+// rows n+8b .. n+8b+7 and needs k in [n-1, top_b - 1], i.e. ceil((8b+8)/64) =
+// b/8 + 1 chunks of 64. Tiles are numbered group by group (blocks 8g..8g+7 have
+// g+1 chunks each, 4g(g+1) tiles precede group g) and dealt round-robin to the
+// CTA's threads; each tile's 8 partial minima are combined with atomicMin.
+template <typename T, bool FWD>
+__device__ __forceinline__ void fill_tiles(int L, int n, T dtv, const T *S, const T *Rb,
+                                           const T *prev, T *best)
+{
+    const int t = threadIdx.x, nt = blockDim.x;
+    const T ndt = T(T(n) * dtv);
+    const int nb = (L - n + 1 + kRB - 1) / kRB;
+    const int ng = (nb + 7) / 8;
+    const int ntiles = 4 * ng * (ng + 1);
+    for (int q = t; q < ntiles; q += nt) {
+        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
+        while (4 * (g + 1) * (g + 2) <= q) ++g;
+        while (g > 0 && 4 * g * (g + 1) > q) --g;
+        const int r = q - 4 * g * (g + 1);
+        const int b = 8 * g + r / (g + 1);
+        const int j = r % (g + 1);
+        if (b >= nb) continue;
+        const int bot = n + kRB * b;
+        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
+        const int k0 = n - 1 + kKC * j;
+        if (k0 > top - 1) continue;
+        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        T R[kRB], acc[kRB];
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj) {
+            const int m = bot + jj <= top ? bot + jj : top;
+            R[jj] = FWD ? T(ndt + Rb[skew(m)]) : Rb[skew(m)];
+            acc[jj] = T(~T(0));
+        }
+        const int kf = k1 < bot ? k1 : bot;  // k < bot: every row of the block takes it
+        for (int k = k0; k < kf; ++k) {
+            const T v = prev[skew(k)], sk = S[skew(k)];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) acc[jj] = dmin(acc[jj], T(dmax(v, R[jj]) - sk));
+        }
+        if (k1 > bot) {  // row bot+jj takes k < bot+jj
+#pragma unroll
+            for (int u = 0; u < kRB - 1; ++u) {
+                const int k = bot + u;
+                if (k >= k1) break;
+                if (k < k0) continue;
+                const T v = prev[skew(k)], sk = S[skew(k)];
+#pragma unroll
+                for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = dmin(acc[jj], T(dmax(v, R[jj]) - sk));
+            }
+        }
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj)
+            if (bot + jj <= top) atomic_min_T(&best[skew(bot + jj)], acc[jj]);
+    }
+}
+
 template <typename T, bool FWD>
 __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, const uint64_t *P64c,
                       const uint64_t *P64x, unsigned char *arrays, uint32_t *bitsw,
                       T *table)
 {
-    const int L = a.L, t = threadIdx.x, nt = blockDim.x;
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
     T *S = reinterpret_cast<T *>(arrays);
-    T *Rb = S + (L + 1);
-    T *colA = Rb + (L + 1);
-    T *colB = colA + (L + 1);
+    T *Rb = S + Ls;
+    T *colA = Rb + Ls;
+    T *colB = colA + Ls;
+    T *best = colB + Ls;
     // P64c / P64x sit in the 64-bit column-buffer bytes, past the typed S and R
     // arrays for either T; the typed columns overwrite them only after this copy.
     for (int m = t; m <= L; m += nt) {
-        S[m] = T(FWD ? P64c[m] : P64x[m]);
-        Rb[m] = T(FWD ? P64x[m] : P64c[m]);
+        S[skew(m)] = T(FWD ? P64c[m] : P64x[m]);
+        Rb[skew(m)] = T(FWD ? P64x[m] : P64c[m]);
     }
     __syncthreads();
 
     const T dtv = T(dti);
     const T c = FWD ? T(0) : dtv;
-    // column 1
-    for (int m = 1 + t; m <= L; m += nt) {
-        const T R = FWD ? T(dtv + Rb[m]) : Rb[m];
-        const T v = T(R + S[m] + c);
-        colA[m] = v;
+    for (int m = 1 + t; m <= L; m += nt) {  // column 1
+        const T R = FWD ? T(dtv + Rb[skew(m)]) : Rb[skew(m)];
+        const T v = T(R + S[skew(m)] + c);
+        colA[skew(m)] = v;
+        best[skew(m)] = T(~T(0));
         table[tri_index(L, m, 1)] = v;
     }
     __syncthreads();
     T *prev = colA, *cur = colB;
     for (int n = 2; n <= L; ++n) {
-        const T ndt = T(T(n) * dtv);
+        fill_tiles<T, FWD>(L, n, dtv, S, Rb, prev, best);
+        __syncthreads();
         const int64_t cbase = tri_col(L, n) - n;
         for (int m = n + t; m <= L; m += nt) {
-            const T R = FWD ? T(ndt + Rb[m]) : Rb[m];
-            T best = T(dmax(prev[n - 1], R) - S[n - 1]);
-            int k = n;
-            for (; k + 3 < m; k += 4) {
-                const T c0 = T(dmax(prev[k], R) - S[k]);
-                const T c1 = T(dmax(prev[k + 1], R) - S[k + 1]);
-                const T c2 = T(dmax(prev[k + 2], R) - S[k + 2]);
-                const T c3 = T(dmax(prev[k + 3], R) - S[k + 3]);
-                best = dmin(best, dmin(dmin(c0, c1), dmin(c2, c3)));
-            }
-            for (; k < m; ++k) best = dmin(best, T(dmax(prev[k], R) - S[k]));
-            const T v = T(best + S[m] + c);
-            cur[m] = v;
+            const T v = T(best[skew(m)] + S[skew(m)] + c);
+            cur[skew(m)] = v;
+            best[skew(m)] = T(~T(0));
             table[cbase + m] = v;
         }
         __syncthreads();
@@ -162,14 +224,14 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, const uint64_t
         int err = 0;
         int m = L, n = s;
         while (n > 1) {
-            const T R = FWD ? T(T(n) * dtv + Rb[m]) : Rb[m];
-            const T target = T(table[tri_index(L, m, n)] - S[m] - c);
+            const T R = FWD ? T(T(n) * dtv + Rb[skew(m)]) : Rb[skew(m)];
+            const T target = T(table[tri_index(L, m, n)] - S[skew(m)] - c);
             const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
             int found = -1;
             for (int k0 = n - 1; k0 < m; k0 += 32) {
                 const int k = k0 + lane;
                 bool match = false;
-                if (k < m) match = T(dmax(table[pbase + k], R) - S[k]) == target;
+                if (k < m) match = T(dmax(table[pbase + k], R) - S[skew(k)]) == target;
                 const unsigned bal = __ballot_sync(0xffffffffu, match);
                 if (bal) {
                     found = k0 + __ffs(bal) - 1;
@@ -198,7 +260,7 @@ template <bool FWD>
 __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    const int L = a.L, t = threadIdx.x, nt = blockDim.x;
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
     const int W = words_for(L);
     unsigned char *arrays = smem;
     uint32_t *bitsw = reinterpret_cast<uint32_t *>(smem + group_arrays_bytes(L));
@@ -208,8 +270,8 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
     unsigned char *slot =
         a.tables ? a.tables + size_t(blockIdx.x) * size_t(tri_cells(L)) * 8 : smem_table;
     // 64-bit prefix arrays live in the column buffers until the typed copy.
-    uint64_t *P64c = reinterpret_cast<uint64_t *>(arrays) + 2 * (L + 1);
-    uint64_t *P64x = P64c + (L + 1);
+    uint64_t *P64c = reinterpret_cast<uint64_t *>(arrays) + 2 * Ls;
+    uint64_t *P64x = P64c + Ls;
 
     const int64_t count = a.list_count ? int64_t(*a.list_count) : a.batch;
     for (int64_t j = blockIdx.x; j < count; j += gridDim.x) {
@@ -273,8 +335,7 @@ int group_threads(int L)
 {
     if (L <= 64) return 64;
     if (L <= 256) return 128;
-    if (L <= 1024) return 256;
-    return 512;
+    return 256;
 }
 
 }  // namespace
