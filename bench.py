@@ -357,42 +357,25 @@ class _Null:
 
 def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     """Profiles in pinned host memory -> H2D -> forward + backward DP -> f_m of
-    both -> D2H of makespans, decisions and segment counts, every step."""
+    both -> D2H of makespans, decisions, segment counts and replays, every step,
+    through dynacomm.HostPipeline (chunked: copies overlap the solves)."""
+    pipe = dc.HostPipeline(B, L, chunks=args.e2e_chunks, device=dev)
     host_in = {k: v.cpu().pin_memory() for k, v in prof.items()}
-    dev_in = {k: torch.empty_like(v) for k, v in prof.items()}
-    rep = {d: torch.empty(B, dtype=torch.int64, device=dev) for d in (0, 1)}
-    host_out = {}
-    for d in (0, 1):
-        for k in ("makespan", "bits", "nseg"):
-            host_out[(d, k)] = torch.empty_like(sched.out[d][k], device="cpu").pin_memory()
-        host_out[(d, "replay")] = torch.empty(B, dtype=torch.int64).pin_memory()
-    h2d = sum(v.numel() * v.element_size() for v in host_in.values())
-    d2h = sum(v.numel() * v.element_size() for v in host_out.values())
-
-    def e2e_step():
-        for k in host_in:
-            dev_in[k].copy_(host_in[k], non_blocking=True)
-        fo = sched.run(0, dev_in["fc"], dev_in["pt"], dev_in["dt"])
-        bo = sched.run(1, dev_in["bc"], dev_in["gt"], dev_in["dt"])
-        assert dc.dc_eval_timeline_batch(B, L, 0, dev_in["fc"], dev_in["pt"], dev_in["dt"],
-                                         fo["bits"], rep[0]) == 0
-        assert dc.dc_eval_timeline_batch(B, L, 1, dev_in["bc"], dev_in["gt"], dev_in["dt"],
-                                         bo["bits"], rep[1]) == 0
-        for d, o in ((0, fo), (1, bo)):
-            for k in ("makespan", "bits", "nseg"):
-                host_out[(d, k)].copy_(o[k], non_blocking=True)
-            host_out[(d, "replay")].copy_(rep[d], non_blocking=True)
-
+    host_out = pipe.host_buffers()
+    h2d, d2h = pipe.bytes_per_run()
     for _ in range(max(args.warmup, 1)):
-        e2e_step()
+        pipe.run(host_in, host_out)
     torch.cuda.synchronize()
+    for d in (0, 1):  # the pipelined results equal the device-resident path's
+        if not torch.equal(host_out[(d, "makespan")], sched.out[d]["makespan"].cpu()):
+            raise RuntimeError("host pipeline disagrees with the device path")
     steps = max(1, min(args.steps, 5))
     barrier()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record()
     for _ in range(steps):
-        e2e_step()
+        pipe.run(host_in, host_out)
     t1.record()
     torch.cuda.synchronize()
     barrier()
@@ -404,8 +387,9 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
         ms = float(t.item())
     return {"value": B * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps,
-            "path": "pinned host profiles -> dc_schedule_forward/backward_batch -> "
-                    "dc_eval_timeline_batch -> pinned host results"}
+            "path": f"pinned host profiles -> dynacomm.HostPipeline ({pipe.chunks} chunks, "
+                    "copies overlapped with dc_schedule_forward/backward_batch and "
+                    "dc_eval_timeline_batch) -> pinned host results"}
 
 
 def main(argv=None):
@@ -420,6 +404,7 @@ def main(argv=None):
                         "small cases")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--e2e-chunks", type=int, default=8)
     args = p.parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)

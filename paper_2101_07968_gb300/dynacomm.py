@@ -252,3 +252,88 @@ def eval_timeline(direction: int, comp, xfer, dt, bits, stream=None):
     _check(dc_eval_timeline_batch(B, L, direction, comp, xfer, dt, bits, out, stream),
            "dc_eval_timeline_batch")
     return out
+
+
+class HostPipeline:
+    """End-to-end scheduling of profiles that live in pinned host memory.
+
+    The batch is cut into `chunks` contiguous pieces. Three CUDA streams overlap
+    the host->device copy of piece c+1 with the forward DP, backward DP and
+    timeline replay of piece c (all through the C ABI on slices of the device
+    buffers), and with the device->host copy of piece c-1's results. Inputs and
+    outputs are dicts of pinned CPU tensors: inputs fc, pt, bc, gt [batch, L] and
+    dt [batch]; outputs, per direction d in (FWD, BWD), (d, "makespan"),
+    (d, "bits"), (d, "nseg"), (d, "replay").
+    """
+
+    IN_KEYS = ("fc", "pt", "bc", "gt", "dt")
+
+    def __init__(self, batch: int, L: int, chunks: int = 8, device="cuda"):
+        import torch
+        self.batch, self.L, self.W = int(batch), int(L), words(L)
+        self.chunks = max(1, min(int(chunks), self.batch))
+        self.bounds = [self.batch * c // self.chunks for c in range(self.chunks + 1)]
+        step = max(b - a for a, b in zip(self.bounds, self.bounds[1:]))
+        self.ws_bytes = dc_schedule_workspace_bytes(step, L)
+        self.workspace = torch.empty(max(self.ws_bytes, 1), dtype=torch.uint8, device=device)
+        B = self.batch
+        self.dev = {k: torch.empty((B, L), dtype=torch.int64, device=device)
+                    for k in ("fc", "pt", "bc", "gt")}
+        self.dev["dt"] = torch.empty(B, dtype=torch.int64, device=device)
+        self.out = {}
+        for d in (FWD, BWD):
+            self.out[(d, "makespan")] = torch.empty(B, dtype=torch.int64, device=device)
+            self.out[(d, "bits")] = torch.empty((B, max(self.W, 1)), dtype=torch.int32,
+                                                device=device)
+            self.out[(d, "nseg")] = torch.empty(B, dtype=torch.int32, device=device)
+            self.out[(d, "replay")] = torch.empty(B, dtype=torch.int64, device=device)
+        self.s_in, self.s_run, self.s_out = (torch.cuda.Stream(device=device) for _ in range(3))
+        self.ev_in = [torch.cuda.Event() for _ in range(self.chunks)]
+        self.ev_run = [torch.cuda.Event() for _ in range(self.chunks)]
+
+    def host_buffers(self):
+        """Pinned host tensors shaped like the outputs."""
+        return {k: torch_empty_pinned_like(v) for k, v in self.out.items()}
+
+    def bytes_per_run(self):
+        h2d = sum(v.numel() * v.element_size() for v in self.dev.values())
+        d2h = sum(v.numel() * v.element_size() for v in self.out.values())
+        return h2d, d2h
+
+    def run(self, host_in: dict, host_out: dict):
+        import torch
+        cur = torch.cuda.current_stream()
+        self.s_in.wait_stream(cur)
+        for c in range(self.chunks):
+            lo, hi = self.bounds[c], self.bounds[c + 1]
+            if hi <= lo:
+                continue
+            n = hi - lo
+            with torch.cuda.stream(self.s_in):
+                for k in self.IN_KEYS:
+                    self.dev[k][lo:hi].copy_(host_in[k][lo:hi], non_blocking=True)
+                self.ev_in[c].record(self.s_in)
+            self.s_run.wait_event(self.ev_in[c])
+            sr = self.s_run.cuda_stream
+            d = {k: v[lo:hi] for k, v in self.dev.items()}
+            o = {k: v[lo:hi] for k, v in self.out.items()}
+            for dr, (ck, xk) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+                fn = dc_schedule_forward_batch if dr == FWD else dc_schedule_backward_batch
+                _check(fn(n, self.L, d[ck], d[xk], d["dt"], o[(dr, "makespan")],
+                          o[(dr, "bits")], o[(dr, "nseg")], None, self.workspace,
+                          self.ws_bytes, sr), "schedule (host pipeline)")
+                _check(dc_eval_timeline_batch(n, self.L, dr, d[ck], d[xk], d["dt"],
+                                              o[(dr, "bits")], o[(dr, "replay")], sr),
+                       "dc_eval_timeline_batch (host pipeline)")
+            self.ev_run[c].record(self.s_run)
+            self.s_out.wait_event(self.ev_run[c])
+            with torch.cuda.stream(self.s_out):
+                for k, v in o.items():
+                    host_out[k][lo:hi].copy_(v, non_blocking=True)
+        cur.wait_stream(self.s_out)
+        cur.wait_stream(self.s_run)
+
+
+def torch_empty_pinned_like(t):
+    import torch
+    return torch.empty(t.shape, dtype=t.dtype).pin_memory()
