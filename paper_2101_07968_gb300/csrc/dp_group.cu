@@ -1,8 +1,9 @@
 // CTA-per-instance DynaComm DP for any 1 <= L <= 4096 (Eq. 8 / Algorithm 3 and
 // Eq. 9 / Algorithm 4), in 32-bit or 64-bit arithmetic per instance.
 //
-// Used for L > 16, and for the L <= 16 instances whose values need 64 bits
-// (the thread-per-instance kernel puts those on a work list).
+// Used for L > 64, and for the instances the thread-per-instance kernels list
+// (64-bit values, or a traceback deeper than they keep). Transfer costs are
+// capped at the total compute first (exact; see the short-L kernel).
 //
 // Same processing-order template as the small kernel:
 //   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
@@ -93,6 +94,29 @@ __device__ __forceinline__ void atomic_min_T(uint64_t *p, uint64_t v)
     atomicMin(reinterpret_cast<unsigned long long *>(p), static_cast<unsigned long long>(v));
 }
 
+// CTA-wide sums of two per-thread values, returned to every thread.
+__device__ void block_sum2_u64(uint64_t &a, uint64_t &b, uint64_t *scratch /* >= 32 */)
+{
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5, nw = (blockDim.x + 31) >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+    }
+    if (lane == 0) {
+        scratch[warp] = a;
+        scratch[16 + warp] = b;
+    }
+    __syncthreads();
+    a = 0;
+    b = 0;
+    for (int w = 0; w < nw; ++w) {
+        a += scratch[w];
+        b += scratch[16 + w];
+    }
+    __syncthreads();
+}
+
 constexpr int kRB = 8;   // rows per tile
 constexpr int kKC = 64;  // k per tile
 
@@ -154,9 +178,9 @@ __device__ __forceinline__ void fill_tiles(int L, int n, T dtv, const T *S, cons
 }
 
 template <typename T, bool FWD>
-__device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, const uint64_t *P64c,
-                      const uint64_t *P64x, unsigned char *arrays, uint32_t *bitsw,
-                      T *table)
+__device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift,
+                      const uint64_t *P64c, const uint64_t *P64x, unsigned char *arrays,
+                      uint32_t *bitsw, T *table)
 {
     const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
     T *S = reinterpret_cast<T *>(arrays);
@@ -248,7 +272,7 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, const uint64_t
             n -= 1;
         }
         if (lane == 0) {
-            a.makespan[i] = int64_t(bv);
+            a.makespan[i] = int64_t(uint64_t(bv) + shift);
             if (a.nseg) a.nseg[i] = s;
             if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
         }
@@ -280,6 +304,7 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
         const int64_t *xrow = a.xfer + i * L;
         const int64_t dti = a.dt[i];
         int bad_neg = dti < 0, bad_big = (dti >> 52) != 0;
+        uint64_t sc = 0, sx = 0;
         for (int r = 1 + t; r <= L; r += nt) {
             const int col = FWD ? r - 1 : L - r;
             const int64_t cv = __ldg(crow + col), xv = __ldg(xrow + col);
@@ -287,6 +312,8 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
             bad_big |= ((cv | xv) >> 52) != 0;
             P64c[r] = uint64_t(cv);
             P64x[r] = uint64_t(xv);
+            sc += uint64_t(cv);
+            sx += uint64_t(xv);
         }
         for (int w = t; w < W; w += nt) bitsw[w] = 0u;
         if (t == 0) {
@@ -297,18 +324,29 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
         const int any_big = __syncthreads_or(bad_big);
         int st = DC_OK;
         bool narrow = false;
+        uint64_t shift = 0;
         if (any_neg) {
             st = DC_ERR_NEGATIVE;
         } else if (any_big) {
             st = DC_ERR_RANGE;
         } else {
-            block_prefix_u64(P64c, L, scratch);
-            block_prefix_u64(P64x, L, scratch);
-            const uint64_t tc = P64c[L], tx = P64x[L];
-            if (exceeds_range(L, dti, tc, tx))
+            block_sum2_u64(sc, sx, scratch);  // raw totals (each term < 2^52, L <= 4096)
+            if (exceeds_range(L, dti, sc, sx)) {
                 st = DC_ERR_RANGE;
-            else
-                narrow = tc + tx + uint64_t(L) * uint64_t(dti) <= kNarrowLimit;
+            } else {
+                // cap the transfer costs at the total compute: no decision changes,
+                // the makespan drops by sum(xfer) - sum(capped xfer)
+                uint64_t cx = 0, unused = 0;
+                for (int r = 1 + t; r <= L; r += nt) {
+                    P64x[r] = P64x[r] < sc ? P64x[r] : sc;
+                    cx += P64x[r];
+                }
+                block_sum2_u64(cx, unused, scratch);
+                shift = sx - cx;
+                block_prefix_u64(P64c, L, scratch);
+                block_prefix_u64(P64x, L, scratch);
+                narrow = sc + cx + uint64_t(L) * uint64_t(dti) <= kNarrowLimit;
+            }
         }
         if (st != DC_OK) {
             if (t == 0) {
@@ -321,10 +359,10 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
             continue;
         }
         if (narrow)
-            solve<uint32_t, FWD>(a, i, dti, P64c, P64x, arrays, bitsw,
+            solve<uint32_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                                  reinterpret_cast<uint32_t *>(slot));
         else
-            solve<uint64_t, FWD>(a, i, dti, P64c, P64x, arrays, bitsw,
+            solve<uint64_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                                  reinterpret_cast<uint64_t *>(slot));
         for (int w = t; w < W; w += nt) a.bits[i * W + w] = bitsw[w];
         __syncthreads();

@@ -13,6 +13,8 @@
 //    kB transitions (max, subtract, min). Rows are visited top-down so that the
 //    column is updated in place: a block reads only rows below its own top,
 //    which still hold column n-1;
+//  * transfer costs capped at the total compute (exact, as in the short-L
+//    kernel), so that 32-bit values suffice for nearly every instance;
 //  * value-only fill with deferred argmin, as in the short-L kernel: columns
 //    2..kKeep are written to a per-thread slot of the caller's workspace (L2
 //    resident, coalesced across the warp) and the traceback re-derives each
@@ -68,24 +70,21 @@ __global__ void __launch_bounds__(32)
         const int64_t i = int64_t(tile) * 32 + lane;
         if (i >= batch) continue;
 
-        // ---- row -> 32-bit prefix sums in processing order, input checks
+        // ---- row -> 32-bit prefix sums in processing order, input checks; the
+        // transfer costs are capped at the total compute (exact: same decisions,
+        // makespan lower by sum(xfer) - sum(capped xfer), added back below)
         const int64_t *crow = comp + i * L, *xrow = xfer + i * L;
         const int64_t dti = __ldg(dt + i);
         bool neg = dti < 0, big = (dti >> 52) != 0;
-        uint64_t pc = 0, px = 0;
-        lw[0] = 0u;
-        lw[32 * oR] = 0u;
-        for (int r = 1; r <= L; ++r) {
-            const int col = FWD ? r - 1 : L - r;
-            const int64_t cv = __ldg(crow + col), xv = __ldg(xrow + col);
+        uint64_t tc = 0, px = 0;
+        for (int l = 0; l < L; ++l) {
+            const int64_t cv = __ldg(crow + l), xv = __ldg(xrow + l);
             neg |= (cv < 0) | (xv < 0);
             big |= ((cv | xv) >> 52) != 0;
-            pc += uint64_t(cv);
+            tc += uint64_t(cv);
             px += uint64_t(xv);
-            lw[32 * r] = uint32_t(FWD ? pc : px);         // S
-            lw[32 * (oR + r)] = uint32_t(FWD ? px : pc);  // R base
         }
-        if (neg || big || exceeds_range(L, dti, pc, px)) {
+        if (neg || big || exceeds_range(L, dti, tc, px)) {
             const int st = neg ? DC_ERR_NEGATIVE : DC_ERR_RANGE;
             makespan[i] = -int64_t(st);
             if (nseg) nseg[i] = 0;
@@ -93,7 +92,19 @@ __global__ void __launch_bounds__(32)
             for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
             continue;
         }
-        if (pc + px + uint64_t(L) * uint64_t(dti) > kNarrowLimit) {
+        uint64_t pc = 0, pxc = 0;
+        lw[0] = 0u;
+        lw[32 * oR] = 0u;
+        for (int r = 1; r <= L; ++r) {
+            const int col = FWD ? r - 1 : L - r;
+            const uint64_t cv = uint64_t(__ldg(crow + col)), xv = uint64_t(__ldg(xrow + col));
+            pc += cv;
+            pxc += xv < tc ? xv : tc;
+            lw[32 * r] = uint32_t(FWD ? pc : pxc);         // S
+            lw[32 * (oR + r)] = uint32_t(FWD ? pxc : pc);  // R base
+        }
+        const uint64_t shift = px - pxc;
+        if (pc + pxc + uint64_t(L) * uint64_t(dti) > kNarrowLimit) {
             list[atomicAdd(list_count, 1u)] = uint32_t(i);
             continue;
         }
@@ -186,7 +197,7 @@ __global__ void __launch_bounds__(32)
             n -= 1;
             cell = fk;
         }
-        makespan[i] = int64_t(Tbest);
+        makespan[i] = int64_t(uint64_t(Tbest) + shift);
         if (nseg) nseg[i] = s;
         if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
         bits[i * W] = word0;

@@ -21,10 +21,12 @@
 //    the traceback of an s-segment optimum reads columns 1..s-1 only, and s is
 //    small in practice (2-4 on CNN-shaped profiles); an instance whose s needs a
 //    deeper column is re-solved by the 64-bit pass, which keeps every column;
-//  * 32-bit values whenever the instance bound L*dt + sum(xfer) + sum(comp) is
-//    below 2^32 - 1: every DP value and candidate lies in [0, bound], so the
-//    32-bit fill is exact. Other instances (and the deep ones above) are
-//    appended to a work list that a 64-bit instantiation solves afterwards;
+//  * transfer costs are first capped at the instance's total compute, which
+//    changes no decision (see row_prefix); 32-bit values whenever the capped
+//    bound L*dt + sum(capped xfer) + sum(comp) is below 2^32 - 1: every DP value
+//    and candidate lies in [0, bound], so the 32-bit fill is exact. Other
+//    instances (and the deep ones above) are appended to a work list that a
+//    64-bit instantiation solves afterwards;
 //  * persistent warps: each warp walks 32-instance tiles; while it solves one
 //    tile, the next tile's rows stream into a padded shared buffer with
 //    cp.async (coalesced 8-byte copies, odd row stride so that every lane reads
@@ -51,6 +53,10 @@ __host__ __device__ constexpr int cell2(int L, int m, int n)
     return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
 }
 
+// Row stride of the staging buffer in int64 units: odd, so that the 16 lanes of a
+// half-warp reading 64-bit words of their own rows hit 16 distinct bank pairs.
+__host__ __device__ constexpr int stage_stride(int L) { return (L % 2 == 0) ? L + 1 : L; }
+
 // Stored columns 2..C with C = min(keep, L-1); KEEP = L keeps them all.
 template <int L, typename T, int KEEP>
 struct Small {
@@ -60,7 +66,7 @@ struct Small {
     static constexpr int kOffS = kCells;                                // S[0..L]
     static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
     static constexpr int kLaneVals = kCells + 2 * (L + 1);
-    static constexpr int kStride = (L % 2 == 0) ? L + 1 : L;  // staging row stride (int64, odd)
+    static constexpr int kStride = stage_stride(L);          // staging row stride (int64, odd)
     static constexpr int kStageBytes = 2 * 32 * kStride * 8;   // comp + xfer rows of a tile
     static constexpr int kTableBytes = 32 * kLaneVals * int(sizeof(T));
     static constexpr int kWarpBytes = kStageBytes + kTableBytes;
@@ -129,8 +135,9 @@ __device__ __forceinline__ T prev_cell(const T *lw, int k, int nm1, T dtv, T c)
 // pass did not keep; the caller then lists the instance for the full pass.
 template <int L, bool FWD, typename T, int KEEP>
 __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
-                                      int64_t dti, T *lw, int64_t i, int64_t *makespan,
-                                      uint32_t *bits, int32_t *nseg, int32_t *status)
+                                      int64_t dti, uint64_t shift, T *lw, int64_t i,
+                                      int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                                      int32_t *status)
 {
     using K = Small<L, T, KEEP>;
     constexpr int W = (L - 1 + 31) / 32;
@@ -174,7 +181,7 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
         n -= 1;
         cell = fk;
     }
-    makespan[i] = int64_t(Tbest);
+    makespan[i] = int64_t(uint64_t(Tbest) + shift);
     if (nseg) nseg[i] = s;
     if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
     if (W > 0) bits[i * W] = word;
@@ -194,7 +201,7 @@ template <int L>
 __device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int64_t *comp,
                                            const int64_t *xfer, int64_t base, int rows, int lane)
 {
-    constexpr int kStride = Small<L, uint32_t, L>::kStride;
+    constexpr int kStride = stage_stride(L);
     const int64_t *gC = comp + base * L;
     const int64_t *gX = xfer + base * L;
     const int nel = rows * L;
@@ -206,22 +213,35 @@ __device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int
     cp_async_commit();
 }
 
-// Read this lane's row (processing order) into 64-bit prefix sums; flag bad input.
+// Read this lane's row (processing order) into 64-bit prefix sums; flag bad
+// input. Transfer costs are capped at the row's total compute: shifted by
+// n*dt + (transfer prefix), every DP value lies in [0, total compute] and the
+// recurrence sees transfer costs only through saturating differences, so the cap
+// changes no comparison (same decision) and lowers the makespan by exactly
+// sum(xfer) - sum(capped xfer), returned in `shift`.
 template <int L, bool FWD, typename Src>
 __device__ __forceinline__ void row_prefix(Src get, uint64_t (&Pc)[L + 1], uint64_t (&Px)[L + 1],
-                                           bool &neg, bool &big)
+                                           uint64_t &xraw, bool &neg, bool &big)
 {
+    uint64_t tc = 0;
+    xraw = 0;
+#pragma unroll
+    for (int r = 1; r <= L; ++r) {
+        int64_t cv, xv;
+        get(FWD ? r - 1 : L - r, cv, xv);
+        neg |= (cv < 0) | (xv < 0);
+        big |= ((cv | xv) >> 52) != 0;
+        tc += uint64_t(cv);
+        xraw += uint64_t(xv);
+    }
     Pc[0] = 0;
     Px[0] = 0;
 #pragma unroll
     for (int r = 1; r <= L; ++r) {
-        const int col = FWD ? r - 1 : L - r;
         int64_t cv, xv;
-        get(col, cv, xv);
-        neg |= (cv < 0) | (xv < 0);
-        big |= ((cv | xv) >> 52) != 0;
+        get(FWD ? r - 1 : L - r, cv, xv);
         Pc[r] = Pc[r - 1] + uint64_t(cv);
-        Px[r] = Px[r - 1] + uint64_t(xv);
+        Px[r] = Px[r - 1] + (uint64_t(xv) < tc ? uint64_t(xv) : tc);
     }
 }
 
@@ -264,31 +284,29 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         const int64_t dti = active ? __ldg(dt + i) : 0;
         cp_async_wait_all();
         __syncwarp();
-        uint64_t Pc[L + 1], Px[L + 1];
+        uint64_t Pc[L + 1], Px[L + 1], xraw;
         bool neg = dti < 0, big = (dti >> 52) != 0;
         row_prefix<L, FWD>(
             [&](int col, int64_t &cv, int64_t &xv) {
                 cv = active ? stC[lane * K::kStride + col] : 0;
                 xv = active ? stX[lane * K::kStride + col] : 0;
             },
-            Pc, Px, neg, big);
+            Pc, Px, xraw, neg, big);
         __syncwarp();  // staging free: prefetch the next tile under this tile's DP
         const int64_t next = tile + gridDim.x;
         if (next < tiles) stage_tile<L>(stC, stX, comp, xfer, next * 32, rows_of(next), lane);
         if (!active) continue;
         int st = DC_OK;
-        uint64_t bound = 0;
-        if (neg) {
+        if (neg)
             st = DC_ERR_NEGATIVE;
-        } else {
-            bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];
-            if (big || bound >= uint64_t(kRangeLimit)) st = DC_ERR_RANGE;
-        }
+        else if (big || uint64_t(L) * uint64_t(dti) + Pc[L] + xraw >= uint64_t(kRangeLimit))
+            st = DC_ERR_RANGE;
+        const uint64_t bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];  // capped
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
         } else if (bound > kNarrowLimit ||
-                   !solve<L, FWD, uint32_t, kKeepCols>(Pc, Px, dti, lw, i, makespan, bits, nseg,
-                                                       status)) {
+                   !solve<L, FWD, uint32_t, kKeepCols>(Pc, Px, dti, xraw - Px[L], lw, i,
+                                                       makespan, bits, nseg, status)) {
             // 64-bit values, or a traceback deeper than the kept columns: work list
             wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
         }
@@ -315,15 +333,16 @@ __global__ void __launch_bounds__(32)
         const int64_t *crow = comp + i * L;
         const int64_t *xrow = xfer + i * L;
         const int64_t dti = __ldg(dt + i);
-        uint64_t Pc[L + 1], Px[L + 1];
+        uint64_t Pc[L + 1], Px[L + 1], xraw;
         bool neg = false, big = false;  // checked by the dense pass
         row_prefix<L, FWD>(
             [&](int col, int64_t &cv, int64_t &xv) {
                 cv = __ldg(crow + col);
                 xv = __ldg(xrow + col);
             },
-            Pc, Px, neg, big);
-        solve<L, FWD, uint64_t, L>(Pc, Px, dti, lw, i, makespan, bits, nseg, status);
+            Pc, Px, xraw, neg, big);
+        solve<L, FWD, uint64_t, L>(Pc, Px, dti, xraw - Px[L], lw, i, makespan, bits, nseg,
+                                   status);
     }
 }
 

@@ -338,3 +338,29 @@ def test_generator_rejects_bad_config(orc):
         bad[key] = val
         with pytest.raises(ValueError):
             orc.profile_gen(bad)
+
+
+# ------------------------------------------------- transfer-capping invariance
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_capping_transfers_at_total_compute_keeps_decisions(orc, direction):
+    """Shifting each DP value by n*dt + (transfer prefix) leaves a quantity in
+    [0, total compute] whose recurrence sees transfer costs only through
+    saturating differences, so capping every per-layer transfer cost at the total
+    compute changes no candidate comparison: same decision, same segment count,
+    makespan lower by exactly sum(xfer) - sum(capped xfer). The GPU kernels rely
+    on this to solve in 32 bits instances whose raw bound exceeds 2^32."""
+    rng = np.random.default_rng(301 + direction)
+    for trial in range(400):
+        L = int(rng.integers(1, 13))
+        comp = rng.integers(0, 50, size=L)
+        xfer = rng.integers(0, 50, size=L)
+        big = rng.random(L) < 0.4  # heavy-tailed transfers, many above the cap
+        xfer[big] += rng.integers(0, 10_000, size=big.sum())
+        if trial % 7 == 0:
+            comp[:] = 0  # cap 0: every transfer capped to nothing
+        dt = int(rng.integers(0, 60))
+        capped = np.minimum(xfer, comp.sum())
+        v, d, s = orc.dp(direction, comp, xfer, dt)
+        vc, dc_, sc = orc.dp(direction, comp, capped, dt)
+        assert (list(d), s) == (list(dc_), sc), (comp, xfer, dt)
+        assert v - vc == int(xfer.sum() - capped.sum())
