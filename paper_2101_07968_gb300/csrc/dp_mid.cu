@@ -174,18 +174,31 @@ __global__ void __launch_bounds__(32)
             const uint32_t rm = lw[32 * (oR + m)];
             const uint32_t R = FWD ? uint32_t(n) * dtv + rm : rm;
             const uint32_t target = cell - lw[32 * m] - c;
-            int k = n - 1;
+            // candidates in groups of 4 (loads issued together, lowest match wins)
+            int k = -1;
             uint32_t fk = 0;
-            for (; k < m; ++k) {
-                if (n - 1 == 1) {
-                    const uint32_t rb = lw[32 * (oR + k)];
-                    fk = (FWD ? dtv + rb : rb) + lw[32 * k] + c;
-                } else {
-                    fk = myslot[int64_t(mid_cell(L, k, n - 1)) * nslots];
+            for (int k0 = n - 1; k0 < m && k < 0; k0 += 4) {
+                uint32_t f[4], sk[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
+                    if (n - 1 == 1) {
+                        const uint32_t rb = lw[32 * (oR + kk)];
+                        f[u] = (FWD ? dtv + rb : rb) + lw[32 * kk] + c;
+                    } else {
+                        f[u] = myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots];
+                    }
+                    sk[u] = lw[32 * kk];
                 }
-                if (dmax(fk, R) - lw[32 * k] == target) break;
+#pragma unroll
+                for (int u = 3; u >= 0; --u) {
+                    if (k0 + u < m && dmax(f[u], R) - sk[u] == target) {
+                        k = k0 + u;
+                        fk = f[u];
+                    }
+                }
             }
-            if (k >= m) {
+            if (k < 0) {
                 err = 1;
                 break;
             }

@@ -45,6 +45,7 @@ namespace {
 #ifndef DC_TREE_MIN
 #define DC_TREE_MIN 1
 #endif
+constexpr int kTbGroup = 4;  // traceback candidates loaded per round
 constexpr int kKeepCols = DC_KEEP_COLS;  // the 32-bit pass stores columns 2..kKeepCols
 
 // index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
@@ -166,13 +167,27 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
         const T rm = lds(lw, K::kOffR + m);
         const T R = FWD ? T(T(n) * dtv + rm) : rm;
         const T target = T(cell - lds(lw, K::kOffS + m) - c);
-        int k = n - 1;
+        // candidates in groups of kTbGroup: the loads issue back to back, then the
+        // compares run from the highest k down so that the lowest match wins
+        int k = -1;
         T fk = T(0);
-        for (; k < m; ++k) {
-            fk = prev_cell<L, FWD, T, KEEP>(lw, k, n - 1, dtv, c);
-            if (T(dmax(fk, R) - lds(lw, K::kOffS + k)) == target) break;
+        for (int k0 = n - 1; k0 < m && k < 0; k0 += kTbGroup) {
+            T f[kTbGroup], sk[kTbGroup];
+#pragma unroll
+            for (int u = 0; u < kTbGroup; ++u) {
+                const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
+                f[u] = prev_cell<L, FWD, T, KEEP>(lw, kk, n - 1, dtv, c);
+                sk[u] = lds(lw, K::kOffS + kk);
+            }
+#pragma unroll
+            for (int u = kTbGroup - 1; u >= 0; --u) {
+                if (k0 + u < m && T(dmax(f[u], R) - sk[u]) == target) {
+                    k = k0 + u;
+                    fk = f[u];
+                }
+            }
         }
-        if (k >= m) {  // cannot happen: the fill and this check use the same arithmetic
+        if (k < 0) {  // cannot happen: the fill and this check use the same arithmetic
             err = 1;
             break;
         }
