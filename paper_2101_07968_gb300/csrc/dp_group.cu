@@ -280,8 +280,175 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
     __syncthreads();
 }
 
+// ---------------------------------------------------------------------------
+// Backward direction in 32 bits for instances whose (capped) bound exceeds 2^32.
+// Shift every value by n*dt + GTR[m] (the link's own work):
+//   E[m][n] = B[m][n] - n*dt - GTR[m]  lies in [0, BCR[m]]
+// and Eq. 9 becomes
+//   E[m][n] = min_{k} max(E[k][n-1], BCR[m] - ((n-1)*dt + GTR[k])),  E[m][1] = BCR[m].
+// The second term only matters when positive (E >= 0), so (n-1)*dt + GTR[k] may be
+// clamped to 2^31 - 1: with total backward compute below 2^31 every quantity fits
+// a signed 32-bit word and a transition is again subtract, max, min. Candidates
+// of a cell differ from Eq. 9's by the row constant n*dt + GTR[m], so every
+// argmin (and the lowest-k rule) is unchanged; B[L][n] = E[L][n] + n*dt + GTR[L].
+constexpr int32_t kYClamp = 0x7fffffff;
+
+__device__ __forceinline__ int32_t yclamp(uint64_t v) { return v < uint64_t(kYClamp) ? int32_t(v) : kYClamp; }
+
+__device__ __forceinline__ void fill_tiles_ebwd(int L, int n, const int32_t *BC, const int32_t *Y,
+                                                const int32_t *prev, int32_t *best)
+{
+    const int t = threadIdx.x, nt = blockDim.x;
+    const int nb = (L - n + 1 + kRB - 1) / kRB;
+    const int ng = (nb + 7) / 8;
+    const int ntiles = 4 * ng * (ng + 1);
+    for (int q = t; q < ntiles; q += nt) {
+        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
+        while (4 * (g + 1) * (g + 2) <= q) ++g;
+        while (g > 0 && 4 * g * (g + 1) > q) --g;
+        const int r = q - 4 * g * (g + 1);
+        const int b = 8 * g + r / (g + 1);
+        const int j = r % (g + 1);
+        if (b >= nb) continue;
+        const int bot = n + kRB * b;
+        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
+        const int k0 = n - 1 + kKC * j;
+        if (k0 > top - 1) continue;
+        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        int32_t R[kRB], acc[kRB];
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj) {
+            const int m = bot + jj <= top ? bot + jj : top;
+            R[jj] = BC[skew(m)];
+            acc[jj] = 0x7fffffff;
+        }
+        const int kf = k1 < bot ? k1 : bot;
+        for (int k = k0; k < kf; ++k) {
+            const int32_t v = prev[skew(k)], y = Y[skew(k)];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(v, R[jj] - y));
+        }
+        if (k1 > bot) {
+#pragma unroll
+            for (int u = 0; u < kRB - 1; ++u) {
+                const int k = bot + u;
+                if (k >= k1) break;
+                if (k < k0) continue;
+                const int32_t v = prev[skew(k)], y = Y[skew(k)];
+#pragma unroll
+                for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(v, R[jj] - y));
+            }
+        }
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj)
+            if (bot + jj <= top) atomicMin(&best[skew(bot + jj)], acc[jj]);
+    }
+}
+
+__device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift,
+                           const uint64_t *P64c, const uint64_t *P64x, unsigned char *arrays,
+                           uint32_t *bitsw, int32_t *table)
+{
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
+    // bytes [0, 8Ls): GTR (64-bit); then BCR, two columns, partial minima, Y (32-bit).
+    // P64c / P64x occupy bytes [16Ls, 32Ls): read before anything past 16Ls is written.
+    uint64_t *GT = reinterpret_cast<uint64_t *>(arrays);
+    int32_t *BC = reinterpret_cast<int32_t *>(arrays + size_t(8) * Ls);
+    int32_t *colA = BC + Ls;
+    int32_t *colB = colA + Ls;
+    int32_t *best = colB + Ls;
+    int32_t *Y = best + Ls;
+    for (int m = t; m <= L; m += nt) {
+        GT[skew(m)] = P64x[m];
+        BC[skew(m)] = int32_t(P64c[m]);
+    }
+    __syncthreads();
+    const uint64_t dtv = uint64_t(dti);
+    for (int m = 1 + t; m <= L; m += nt) {  // column 1, and Y for column 2
+        const int32_t v = BC[skew(m)];
+        colA[skew(m)] = v;
+        best[skew(m)] = 0x7fffffff;
+        table[tri_index(L, m, 1)] = v;
+        Y[skew(m)] = yclamp(dtv + GT[skew(m)]);
+    }
+    __syncthreads();
+    int32_t *prev = colA, *cur = colB;
+    for (int n = 2; n <= L; ++n) {
+        fill_tiles_ebwd(L, n, BC, Y, prev, best);
+        __syncthreads();
+        const int64_t cbase = tri_col(L, n) - n;
+        for (int m = n + t; m <= L; m += nt) {
+            const int32_t v = best[skew(m)];
+            cur[skew(m)] = v;
+            best[skew(m)] = 0x7fffffff;
+            table[cbase + m] = v;
+        }
+        for (int k = n + t; k <= L; k += nt) Y[skew(k)] = yclamp(uint64_t(n) * dtv + GT[skew(k)]);
+        __syncthreads();
+        int32_t *tmp = prev;
+        prev = cur;
+        cur = tmp;
+    }
+    if (t < 32) {
+        const int lane = t;
+        uint64_t bv = ~uint64_t(0);  // E[L][n] + n*dt: B[L][n] less the constant GTR[L]
+        int bn = 0x7fffffff;
+        for (int n = 1 + lane; n <= L; n += 32) {
+            const uint64_t v = uint64_t(table[tri_index(L, L, n)]) + uint64_t(n) * dtv;
+            if (v < bv) {
+                bv = v;
+                bn = n;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const uint64_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int on = __shfl_xor_sync(0xffffffffu, bn, o);
+            if (ov < bv || (ov == bv && on < bn)) {
+                bv = ov;
+                bn = on;
+            }
+        }
+        const int s = bn;
+        int err = 0, m = L, n = s;
+        while (n > 1) {
+            const int32_t R = BC[skew(m)];
+            const int32_t target = table[tri_index(L, m, n)];
+            const int64_t pbase = tri_col(L, n - 1) - (n - 1);
+            int found = -1;
+            for (int k0 = n - 1; k0 < m; k0 += 32) {
+                const int k = k0 + lane;
+                bool match = false;
+                if (k < m) {
+                    const int32_t y = yclamp(uint64_t(n - 1) * dtv + GT[skew(k)]);
+                    match = max(table[pbase + k], R - y) == target;
+                }
+                const unsigned bal = __ballot_sync(0xffffffffu, match);
+                if (bal) {
+                    found = k0 + __ffs(bal) - 1;
+                    break;
+                }
+            }
+            if (found < 0) {
+                err = 1;
+                break;
+            }
+            if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
+            __syncwarp();
+            m = found;
+            n -= 1;
+        }
+        if (lane == 0) {
+            a.makespan[i] = int64_t(bv + GT[skew(L)] + shift);
+            if (a.nseg) a.nseg[i] = s;
+            if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+        }
+    }
+    __syncthreads();
+}
+
 template <bool FWD>
-__global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
+__global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
@@ -361,6 +528,9 @@ __global__ void __launch_bounds__(512) group_kernel(GroupArgs a)
         if (narrow)
             solve<uint32_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                                  reinterpret_cast<uint32_t *>(slot));
+        else if (!FWD && sc < uint64_t(kYClamp))
+            solve_ebwd(a, i, dti, shift, P64c, P64x, arrays, bitsw,
+                       reinterpret_cast<int32_t *>(slot));
         else
             solve<uint64_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                                  reinterpret_cast<uint64_t *>(slot));

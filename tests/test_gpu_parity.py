@@ -79,7 +79,7 @@ def test_dp_random_parity(dc, L, kind):
         _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
 
 
-@pytest.mark.parametrize("L", [1, 2, 8, 16, 17, 54, 70])
+@pytest.mark.parametrize("L", [1, 2, 8, 16, 17, 54, 70, 100, 200])
 def test_dp_wide_values_parity(dc, L):
     """Instances whose bound exceeds 2^32 need 64-bit arithmetic; mix them with
     32-bit ones so both paths (and the work list) run in one call."""
