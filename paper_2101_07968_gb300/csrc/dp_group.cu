@@ -447,6 +447,205 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
     __syncthreads();
 }
 
+// ---------------------------------------------------------------------------
+// Forward direction in 32 bits for instances whose (capped) bound exceeds 2^32.
+// Shift every value by n*dt + P[m] (the arrival time of the last pull):
+//   E[m][n] = F[m][n] - n*dt - P[m]  lies in [0, FC[m]]
+// and, with G[k] = FC[L] - FC[k], A[k] = E[k][n-1] + G[k] + P[k], Q[m] = dt + P[m],
+// Eq. 8 becomes
+//   E[m][n] + G[m] = min_{k} max(A[k] - Q[m], G[k]),  E[m][1] = FC[m].
+// A[k] and Q[m] are large but only a non-negative difference below 2^30 matters,
+// so inside a tile both are taken relative to P at the tile's lowest row: when
+// the tile's rows span less than 2^30 of transfer, A - P[bot] clamped below at
+// -2^30 and Q - P[bot] are signed 32-bit and the transition is subtract, max,
+// min; other tiles use the same formula in 64-bit. Candidates differ from Eq. 8's
+// by the row constant n*dt + P[m] + G[m]: every argmin is unchanged, and
+// F[L][n] = E[L][n] + n*dt + P[L]. Needs FC[L] < 2^29.
+constexpr int32_t kSpan = 1 << 30;
+
+__device__ __forceinline__ void fill_tiles_efwd(int L, int n, uint64_t dtv, const uint64_t *P,
+                                                const int32_t *G, const uint64_t *A,
+                                                int32_t *best)
+{
+    const int t = threadIdx.x, nt = blockDim.x;
+    const int nb = (L - n + 1 + kRB - 1) / kRB;
+    const int ng = (nb + 7) / 8;
+    const int ntiles = 4 * ng * (ng + 1);
+    for (int q = t; q < ntiles; q += nt) {
+        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
+        while (4 * (g + 1) * (g + 2) <= q) ++g;
+        while (g > 0 && 4 * g * (g + 1) > q) --g;
+        const int r = q - 4 * g * (g + 1);
+        const int b = 8 * g + r / (g + 1);
+        const int j = r % (g + 1);
+        if (b >= nb) continue;
+        const int bot = n + kRB * b;
+        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
+        const int k0 = n - 1 + kKC * j;
+        if (k0 > top - 1) continue;
+        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        const int kf = k1 < bot ? k1 : bot;
+        const uint64_t base = P[skew(bot)];
+        int32_t acc[kRB];
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj) acc[jj] = 0x7fffffff;
+        if (dtv + (P[skew(top)] - base) < uint64_t(kSpan)) {
+            int32_t Qr[kRB];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) {
+                const int m = bot + jj <= top ? bot + jj : top;
+                Qr[jj] = int32_t(dtv + (P[skew(m)] - base));
+            }
+            for (int k = k0; k < kf; ++k) {
+                const int64_t ad = int64_t(A[skew(k)] - base);
+                const int32_t a = ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
+                const int32_t gk = G[skew(k)];
+#pragma unroll
+                for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(a - Qr[jj], gk));
+            }
+            if (k1 > bot) {
+#pragma unroll
+                for (int u = 0; u < kRB - 1; ++u) {
+                    const int k = bot + u;
+                    if (k >= k1) break;
+                    if (k < k0) continue;
+                    const int64_t ad = int64_t(A[skew(k)] - base);
+                    const int32_t a = ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
+                    const int32_t gk = G[skew(k)];
+#pragma unroll
+                    for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(a - Qr[jj], gk));
+                }
+            }
+        } else {  // wide tile: the same candidates in 64-bit
+            int64_t Qw[kRB];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) {
+                const int m = bot + jj <= top ? bot + jj : top;
+                Qw[jj] = int64_t(dtv + P[skew(m)]);
+            }
+            for (int k = k0; k < k1; ++k) {
+                const int64_t ak = int64_t(A[skew(k)]);
+                const int64_t gk = G[skew(k)];
+#pragma unroll
+                for (int jj = 0; jj < kRB; ++jj)
+                    if (k < bot + jj) {
+                        const int64_t x = ak - Qw[jj];
+                        acc[jj] = min(acc[jj], int32_t(x > gk ? x : gk));
+                    }
+            }
+        }
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj)
+            if (bot + jj <= top) atomicMin(&best[skew(bot + jj)], acc[jj]);
+    }
+}
+
+__device__ void solve_efwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift,
+                           const uint64_t *P64c, const uint64_t *P64x, unsigned char *arrays,
+                           uint32_t *bitsw, int32_t *table)
+{
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
+    // bytes [0, 8Ls): P (64-bit), [8Ls, 12Ls): G, [12Ls, 16Ls): column A,
+    // [16Ls, 24Ls): A (64-bit), [24Ls, 28Ls): column B, [28Ls, 32Ls): partial minima.
+    // P64c / P64x occupy bytes [16Ls, 32Ls): only P and G are written before the barrier.
+    uint64_t *P = reinterpret_cast<uint64_t *>(arrays);
+    int32_t *G = reinterpret_cast<int32_t *>(arrays + size_t(8) * Ls);
+    int32_t *colA = G + Ls;
+    uint64_t *A = reinterpret_cast<uint64_t *>(arrays + size_t(16) * Ls);
+    int32_t *colB = reinterpret_cast<int32_t *>(arrays + size_t(24) * Ls);
+    int32_t *best = colB + Ls;
+    const uint64_t fcL = P64c[L];
+    for (int m = t; m <= L; m += nt) {
+        P[skew(m)] = P64x[m];
+        G[skew(m)] = int32_t(fcL - P64c[m]);
+    }
+    __syncthreads();
+    const uint64_t dtv = uint64_t(dti);
+    for (int m = 1 + t; m <= L; m += nt) {  // column 1: E = FC[m]; A for column 2
+        const int32_t v = int32_t(fcL) - G[skew(m)];
+        colA[skew(m)] = v;
+        best[skew(m)] = 0x7fffffff;
+        table[tri_index(L, m, 1)] = v;
+        A[skew(m)] = fcL + P[skew(m)];
+    }
+    __syncthreads();
+    int32_t *prev = colA, *cur = colB;
+    for (int n = 2; n <= L; ++n) {
+        fill_tiles_efwd(L, n, dtv, P, G, A, best);
+        __syncthreads();
+        const int64_t cbase = tri_col(L, n) - n;
+        for (int m = n + t; m <= L; m += nt) {
+            const int32_t bm = best[skew(m)];
+            const int32_t v = bm - G[skew(m)];
+            cur[skew(m)] = v;
+            best[skew(m)] = 0x7fffffff;
+            table[cbase + m] = v;
+            A[skew(m)] = uint64_t(bm) + P[skew(m)];  // E + G + P for column n+1
+        }
+        __syncthreads();
+        int32_t *tmp = prev;
+        prev = cur;
+        cur = tmp;
+    }
+    if (t < 32) {
+        const int lane = t;
+        uint64_t bv = ~uint64_t(0);  // E[L][n] + n*dt: F[L][n] less the constant P[L]
+        int bn = 0x7fffffff;
+        for (int n = 1 + lane; n <= L; n += 32) {
+            const uint64_t v = uint64_t(table[tri_index(L, L, n)]) + uint64_t(n) * dtv;
+            if (v < bv) {
+                bv = v;
+                bn = n;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const uint64_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int on = __shfl_xor_sync(0xffffffffu, bn, o);
+            if (ov < bv || (ov == bv && on < bn)) {
+                bv = ov;
+                bn = on;
+            }
+        }
+        const int s = bn;
+        int err = 0, m = L, n = s;
+        while (n > 1) {
+            const int64_t Q = int64_t(dtv + P[skew(m)]);
+            const int64_t target = int64_t(table[tri_index(L, m, n)]) + G[skew(m)];
+            const int64_t pbase = tri_col(L, n - 1) - (n - 1);
+            int found = -1;
+            for (int k0 = n - 1; k0 < m; k0 += 32) {
+                const int k = k0 + lane;
+                bool match = false;
+                if (k < m) {
+                    const int64_t gk = G[skew(k)];
+                    const int64_t x = int64_t(table[pbase + k]) + gk + int64_t(P[skew(k)]) - Q;
+                    match = (x > gk ? x : gk) == target;
+                }
+                const unsigned bal = __ballot_sync(0xffffffffu, match);
+                if (bal) {
+                    found = k0 + __ffs(bal) - 1;
+                    break;
+                }
+            }
+            if (found < 0) {
+                err = 1;
+                break;
+            }
+            if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
+            __syncwarp();
+            m = found;
+            n -= 1;
+        }
+        if (lane == 0) {
+            a.makespan[i] = int64_t(bv + P[skew(L)] + shift);
+            if (a.nseg) a.nseg[i] = s;
+            if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+        }
+    }
+    __syncthreads();
+}
+
 template <bool FWD>
 __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
 {
@@ -530,6 +729,9 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
                                  reinterpret_cast<uint32_t *>(slot));
         else if (!FWD && sc < uint64_t(kYClamp))
             solve_ebwd(a, i, dti, shift, P64c, P64x, arrays, bitsw,
+                       reinterpret_cast<int32_t *>(slot));
+        else if (FWD && sc < uint64_t(1) << 29)
+            solve_efwd(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                        reinterpret_cast<int32_t *>(slot));
         else
             solve<uint64_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,

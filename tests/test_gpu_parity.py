@@ -97,6 +97,31 @@ def test_dp_wide_values_parity(dc, L):
         _check_direction(dc, d, comp, xfer, dt, f"wide L={L} dir={d}")
 
 
+@pytest.mark.parametrize("L", [17, 40, 64, 65, 100, 257])
+def test_dp_wide_latency_small_compute_parity(dc, L):
+    """Bound above 2^32 from the latency and the transfers while the total compute
+    stays below 2^29: the shifted 32-bit solves of the per-instance kernel. Thirds
+    of the batch: a huge latency (every 8-row block wider than 2^30 of transfer
+    plus latency); log-uniform transfers with a latency near 2^32 / L (blocks on
+    both sides of 2^30); plain 32-bit instances."""
+    B = 3 * 97 + 5
+    comp, xfer, dt = wl.skewed_instances(313 + L, B, L)
+    rng = np.random.default_rng(1000 + L)
+    part = np.arange(B) % 3
+    comp = comp % (1 << 20)
+    big_dt = part == 0
+    dt[big_dt] = rng.integers(1 << 30, 1 << 40, size=big_dt.sum())
+    big_x = part == 1
+    nb = int(big_x.sum())
+    comp[big_x] = rng.integers((1 << 27) // L, (1 << 29) // L, size=(nb, L))
+    xfer[big_x] = np.exp2(rng.uniform(16, 31, size=(nb, L))).astype(np.int64)
+    dt[big_x] = rng.integers((1 << 31) // L, (1 << 33) // L, size=nb)
+    bound = L * dt + comp.sum(1) + xfer.sum(1)
+    assert (bound[part < 2] > 2**32).all() and (comp.sum(1) < 2**29).all()
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, f"wide-latency L={L} dir={d}")
+
+
 @pytest.mark.parametrize("L", [8, 16, 54, 100])
 def test_dp_status_faults_per_instance(dc, L):
     B = 300
