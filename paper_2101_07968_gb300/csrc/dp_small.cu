@@ -27,10 +27,14 @@
 //    and candidate lies in [0, bound], so the 32-bit fill is exact. Other
 //    instances (and the deep ones above) are appended to a work list that a
 //    64-bit instantiation solves afterwards;
-//  * persistent warps: each warp walks 32-instance tiles; while it solves one
-//    tile, the next tile's rows stream into a padded shared buffer with
-//    cp.async (coalesced 8-byte copies, odd row stride so that every lane reads
-//    its own row without bank conflicts).
+//  * persistent warps: each warp walks 32-instance tiles. A tile's rows arrive
+//    by cp.async (coalesced 8-byte copies) in the warp's own table area, with
+//    an odd row stride so that every lane reads its own row without bank
+//    conflicts; the prefix sums then leave them in registers and the table
+//    overwrites them. Sharing the area keeps a warp at the table's size of
+//    shared memory, so 16 warps fit on an SM (the register limit at <= 128
+//    registers): more resident warps hide more latency than a separate
+//    prefetch buffer would.
 #include "common.cuh"
 
 namespace dc {
@@ -40,7 +44,7 @@ namespace {
 #define DC_KEEP_COLS 4
 #endif
 #ifndef DC_SMALL_MINB
-#define DC_SMALL_MINB 1
+#define DC_SMALL_MINB 16  // resident single-warp CTAs per SM the registers must allow
 #endif
 #ifndef DC_TREE_MIN
 #define DC_TREE_MIN 1
@@ -63,14 +67,14 @@ template <int L, typename T, int KEEP>
 struct Small {
     static constexpr int kLast = KEEP < L - 1 ? KEEP : L - 1;  // last stored column
     static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
-    static constexpr int kW = sizeof(T) / 4;                            // words per value
     static constexpr int kOffS = kCells;                                // S[0..L]
     static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
     static constexpr int kLaneVals = kCells + 2 * (L + 1);
     static constexpr int kStride = stage_stride(L);          // staging row stride (int64, odd)
     static constexpr int kStageBytes = 2 * 32 * kStride * 8;   // comp + xfer rows of a tile
     static constexpr int kTableBytes = 32 * kLaneVals * int(sizeof(T));
-    static constexpr int kWarpBytes = kStageBytes + kTableBytes;
+    // staging and table share the warp's area
+    static constexpr int kWarpBytes = kStageBytes > kTableBytes ? kStageBytes : kTableBytes;
 };
 
 template <typename T>
@@ -269,7 +273,7 @@ __device__ __forceinline__ void write_failure(int st, int64_t i, int W, int64_t 
     for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
 }
 
-// 32-bit pass over the whole batch; persistent warps, cp.async-prefetched tiles.
+// 32-bit pass over the whole batch; persistent warps, tiles staged in the table area.
 template <int L, bool FWD>
 __global__ void __launch_bounds__(32, DC_SMALL_MINB)
     small_dense_kernel(int64_t batch, const int64_t *__restrict__ comp,
@@ -284,16 +288,17 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
     const int lane = threadIdx.x;
     int64_t *stC = reinterpret_cast<int64_t *>(smem);
     int64_t *stX = stC + 32 * K::kStride;
-    uint32_t *lw = reinterpret_cast<uint32_t *>(smem + K::kStageBytes) + lane;
+    uint32_t *lw = reinterpret_cast<uint32_t *>(smem) + lane;
 
     const int64_t tiles = (batch + 31) / 32;
     int64_t tile = blockIdx.x;
     if (tile >= tiles) return;
     auto rows_of = [&](int64_t t) { return int(batch - t * 32 < 32 ? batch - t * 32 : 32); };
-    stage_tile<L>(stC, stX, comp, xfer, tile * 32, rows_of(tile), lane);
     for (; tile < tiles; tile += gridDim.x) {
         const int64_t base = tile * 32;
         const int rows = rows_of(tile);
+        __syncwarp();  // every lane is done with the table: stage the tile's rows there
+        stage_tile<L>(stC, stX, comp, xfer, base, rows, lane);
         const int64_t i = base + lane;
         const bool active = lane < rows;
         const int64_t dti = active ? __ldg(dt + i) : 0;
@@ -307,9 +312,7 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
                 xv = active ? stX[lane * K::kStride + col] : 0;
             },
             Pc, Px, xraw, neg, big);
-        __syncwarp();  // staging free: prefetch the next tile under this tile's DP
-        const int64_t next = tile + gridDim.x;
-        if (next < tiles) stage_tile<L>(stC, stX, comp, xfer, next * 32, rows_of(next), lane);
+        __syncwarp();  // rows read: the lanes' table slices may be written
         if (!active) continue;
         int st = DC_OK;
         if (neg)
@@ -326,7 +329,6 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
             wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
         }
     }
-    cp_async_wait_all();
 }
 
 // 64-bit pass over the work list, every column kept.
