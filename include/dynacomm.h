@@ -196,10 +196,11 @@ const char *dc_status_string(dc_status s);
 
 /* ------------------------------------------------------------------------
  * dc_roof_int_probe -- measurement support, not part of the method: a
- * register-only loop of the DP's per-transition integer operations
- * (variant 0: 32-bit max, subtract, min; variant 1: the same on 64-bit values)
- * on `blocks` x `threads` threads, `iters` iterations of 8 independent
- * transitions each. Time it with events on `stream`; it performs
+ * register-only loop of the DP's per-transition integer operations on
+ * `blocks` x `threads` threads, `iters` iterations of 8 transitions each.
+ * Variant 0: the 32-bit passes' shifted form (one 32-bit add-then-max per
+ * candidate, one 3-input min per two candidates); variant 1: the 64-bit
+ * passes' max, subtract, min. Time it with events on `stream`; it performs
  * blocks*threads*iters*8 transitions. sink: device, blocks*threads uint32.
  * ---------------------------------------------------------------------- */
 dc_status dc_roof_int_probe(int32_t variant, int32_t blocks, int32_t threads, int64_t iters,

@@ -16,6 +16,8 @@ constexpr int kSmemTableLMax = 64;   // group kernel keeps its DP table on chip 
 constexpr int64_t kMidSlots = 152 * 16 * 32;  // traceback slots of the looped kernel
 constexpr int64_t kRangeLimit = int64_t(1) << 52;
 constexpr uint64_t kNarrowLimit = 0xFFFFFFFEull;  // bound that lets a DP run in 32 bits
+// capped bound under which the shifted form of a DP runs in signed 32 bits
+constexpr uint64_t kShiftedLimit = 0x7FFFFFFFull;
 
 // Triangle of DP cells (m, n), 1 <= n <= m <= L, stored column by column:
 // column n holds rows n..L contiguously.

@@ -120,6 +120,26 @@ __device__ void block_sum2_u64(uint64_t &a, uint64_t &b, uint64_t *scratch /* >=
 constexpr int kRB = 8;   // rows per tile
 constexpr int kKC = 64;  // k per tile
 
+// Tile q of column n (numbering below): rows bot..top, candidates k in [k0, k1).
+// Returns false for a tile with no work.
+__device__ __forceinline__ bool decode_tile(int q, int L, int n, int nb, int &bot, int &top,
+                                            int &k0, int &k1)
+{
+    int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
+    while (4 * (g + 1) * (g + 2) <= q) ++g;
+    while (g > 0 && 4 * g * (g + 1) > q) --g;
+    const int r = q - 4 * g * (g + 1);
+    const int b = 8 * g + r / (g + 1);
+    const int j = r % (g + 1);
+    if (b >= nb) return false;
+    bot = n + kRB * b;
+    top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
+    k0 = n - 1 + kKC * j;
+    if (k0 > top - 1) return false;
+    k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+    return true;
+}
+
 // Column n's work is the set of (row block b, k chunk j) tiles: block b holds
 // rows n+8b .. n+8b+7 and needs k in [n-1, top_b - 1], i.e. ceil((8b+8)/64) =
 // b/8 + 1 chunks of 64. Tiles are numbered group by group (blocks 8g..8g+7 have
@@ -135,18 +155,8 @@ __device__ __forceinline__ void fill_tiles(int L, int n, T dtv, const T *S, cons
     const int ng = (nb + 7) / 8;
     const int ntiles = 4 * ng * (ng + 1);
     for (int q = t; q < ntiles; q += nt) {
-        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
-        while (4 * (g + 1) * (g + 2) <= q) ++g;
-        while (g > 0 && 4 * g * (g + 1) > q) --g;
-        const int r = q - 4 * g * (g + 1);
-        const int b = 8 * g + r / (g + 1);
-        const int j = r % (g + 1);
-        if (b >= nb) continue;
-        const int bot = n + kRB * b;
-        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
-        const int k0 = n - 1 + kKC * j;
-        if (k0 > top - 1) continue;
-        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        int bot, top, k0, k1;
+        if (!decode_tile(q, L, n, nb, bot, top, k0, k1)) continue;
         T R[kRB], acc[kRB];
 #pragma unroll
         for (int jj = 0; jj < kRB; ++jj) {
@@ -281,6 +291,182 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
 }
 
 // ---------------------------------------------------------------------------
+// Instances whose capped bound L*dt + sum(comp) + sum(capped xfer) is below 2^31:
+// the shifted form of the thread-per-instance kernels, all in signed 32 bits,
+// where a transition is one add-then-max and two candidates fold with one
+// 3-input min (1.5 integer-ALU instructions per transition):
+//   forward : B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
+//   backward: E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),
+// with G[k] = FC[L] - FC[k], NQ[m] = -(dt + P[m]) (P = transfer prefix),
+// NGT[k] = -(transfer prefix), B[m][1] = FC[L], E[m][1] = BC[m]; U = (NQ, BC) and
+// V = (G, NGT) per direction. The makespan is min_n (B or E)[L][n] + n*dt plus
+// the transfer sum. Each candidate differs from Eq. 8/9's by a constant of its
+// row, so every argmin is unchanged. The table holds A (forward) or E.
+
+template <bool FWD>
+__device__ __forceinline__ int32_t cand_s32(int32_t col, int32_t u, int32_t v)
+{
+    return FWD ? __viaddmax_s32(col, u, v) : __viaddmax_s32(u, v, col);
+}
+
+template <bool FWD>
+__device__ __forceinline__ void fill_tiles_s32(int L, int n, int32_t ndt1, const int32_t *U,
+                                               const int32_t *V, const int32_t *prev,
+                                               int32_t *best)
+{
+    const int t = threadIdx.x, nt = blockDim.x;
+    const int nb = (L - n + 1 + kRB - 1) / kRB;
+    const int ng = (nb + 7) / 8;
+    const int ntiles = 4 * ng * (ng + 1);
+    for (int q = t; q < ntiles; q += nt) {
+        int bot, top, k0, k1;
+        if (!decode_tile(q, L, n, nb, bot, top, k0, k1)) continue;
+        int32_t Ur[kRB], acc[kRB];
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj) {
+            const int m = bot + jj <= top ? bot + jj : top;
+            Ur[jj] = FWD ? U[skew(m)] : U[skew(m)] - ndt1;
+            acc[jj] = 0x7fffffff;
+        }
+        const int kf = k1 < bot ? k1 : bot;  // k < bot: every row of the block takes it
+        int k = k0;
+        for (; k + 1 < kf; k += 2) {
+            const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
+            const int32_t c1 = prev[skew(k + 1)], v1 = V[skew(k + 1)];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj)
+                acc[jj] = __vimin3_s32(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0),
+                                       cand_s32<FWD>(c1, Ur[jj], v1));
+        }
+        if (k < kf) {
+            const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0));
+        }
+        if (k1 > bot) {  // row bot+jj takes k < bot+jj
+#pragma unroll
+            for (int u = 0; u < kRB - 1; ++u) {
+                const int kk = bot + u;
+                if (kk >= k1) break;
+                if (kk < k0) continue;
+                const int32_t c0 = prev[skew(kk)], v0 = V[skew(kk)];
+#pragma unroll
+                for (int jj = u + 1; jj < kRB; ++jj)
+                    acc[jj] = min(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0));
+            }
+        }
+#pragma unroll
+        for (int jj = 0; jj < kRB; ++jj)
+            if (bot + jj <= top) atomicMin(&best[skew(bot + jj)], acc[jj]);
+    }
+}
+
+template <bool FWD>
+__device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t xraw,
+                          const uint64_t *P64c, const uint64_t *P64x, unsigned char *arrays,
+                          uint32_t *bitsw, int32_t *table)
+{
+    const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
+    // bytes [0, 16Ls): U, V, two columns; [16Ls, 20Ls): partial minima. P64c /
+    // P64x occupy bytes [16Ls, 32Ls): only U and V are written before the barrier.
+    int32_t *U = reinterpret_cast<int32_t *>(arrays);
+    int32_t *V = U + Ls;
+    int32_t *colA = V + Ls;
+    int32_t *colB = colA + Ls;
+    int32_t *best = colB + Ls;
+    const int32_t dt = int32_t(dti);
+    const int32_t fcL = int32_t(P64c[L]);
+    for (int m = t; m <= L; m += nt) {
+        U[skew(m)] = FWD ? -(dt + int32_t(P64x[m])) : int32_t(P64c[m]);
+        V[skew(m)] = FWD ? fcL - int32_t(P64c[m]) : -int32_t(P64x[m]);
+    }
+    __syncthreads();
+    for (int m = 1 + t; m <= L; m += nt) {  // column 1
+        const int32_t v = FWD ? fcL - U[skew(m)] - dt : U[skew(m)];
+        colA[skew(m)] = v;
+        best[skew(m)] = 0x7fffffff;
+        table[tri_index(L, m, 1)] = v;
+    }
+    __syncthreads();
+    int32_t *prev = colA, *cur = colB;
+    for (int n = 2; n <= L; ++n) {
+        fill_tiles_s32<FWD>(L, n, (n - 1) * dt, U, V, prev, best);
+        __syncthreads();
+        const int64_t cbase = tri_col(L, n) - n;
+        for (int m = n + t; m <= L; m += nt) {
+            const int32_t b = best[skew(m)];
+            const int32_t v = FWD ? b - U[skew(m)] - dt : b;
+            cur[skew(m)] = v;
+            best[skew(m)] = 0x7fffffff;
+            table[cbase + m] = v;
+        }
+        __syncthreads();
+        int32_t *tmp = prev;
+        prev = cur;
+        cur = tmp;
+    }
+
+    // final pick and traceback by warp 0
+    if (t < 32) {
+        const int lane = t;
+        // (B or E)[L][n] + n*dt, below 2^31
+        const int32_t toB = FWD ? U[skew(L)] + dt : 0;
+        int32_t bv = 0x7fffffff;
+        int bn = 0x7fffffff;
+        for (int n = 1 + lane; n <= L; n += 32) {
+            const int32_t v = table[tri_index(L, L, n)] + toB + n * dt;
+            if (v < bv) {  // n increases: strict keeps the lowest n in this lane
+                bv = v;
+                bn = n;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const int32_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int on = __shfl_xor_sync(0xffffffffu, bn, o);
+            if (ov < bv || (ov == bv && on < bn)) {
+                bv = ov;
+                bn = on;
+            }
+        }
+        const int s = bn;
+        int err = 0;
+        int m = L, n = s;
+        while (n > 1) {
+            const int32_t um = U[skew(m)];
+            const int32_t u = FWD ? um : um - (n - 1) * dt;
+            const int32_t target = table[tri_index(L, m, n)] + (FWD ? um + dt : 0);
+            const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
+            int found = -1;
+            for (int k0 = n - 1; k0 < m; k0 += 32) {
+                const int k = k0 + lane;
+                bool match = false;
+                if (k < m) match = cand_s32<FWD>(table[pbase + k], u, V[skew(k)]) == target;
+                const unsigned bal = __ballot_sync(0xffffffffu, match);
+                if (bal) {
+                    found = k0 + __ffs(bal) - 1;
+                    break;
+                }
+            }
+            if (found < 0) {
+                err = 1;
+                break;
+            }
+            if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
+            __syncwarp();
+            m = found;
+            n -= 1;
+        }
+        if (lane == 0) {
+            a.makespan[i] = int64_t(uint64_t(uint32_t(bv)) + xraw);
+            if (a.nseg) a.nseg[i] = s;
+            if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+        }
+    }
+    __syncthreads();
+}
+
+// ---------------------------------------------------------------------------
 // Backward direction in 32 bits for instances whose (capped) bound exceeds 2^32.
 // Shift every value by n*dt + GTR[m] (the link's own work):
 //   E[m][n] = B[m][n] - n*dt - GTR[m]  lies in [0, BCR[m]]
@@ -288,14 +474,15 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
 //   E[m][n] = min_{k} max(E[k][n-1], BCR[m] - ((n-1)*dt + GTR[k])),  E[m][1] = BCR[m].
 // The second term only matters when positive (E >= 0), so (n-1)*dt + GTR[k] may be
 // clamped to 2^31 - 1: with total backward compute below 2^31 every quantity fits
-// a signed 32-bit word and a transition is again subtract, max, min. Candidates
+// a signed 32-bit word; with NY = -y a transition is one add-then-max and two
+// candidates fold with one 3-input min, as in the 32-bit form above. Candidates
 // of a cell differ from Eq. 9's by the row constant n*dt + GTR[m], so every
 // argmin (and the lowest-k rule) is unchanged; B[L][n] = E[L][n] + n*dt + GTR[L].
 constexpr int32_t kYClamp = 0x7fffffff;
 
 __device__ __forceinline__ int32_t yclamp(uint64_t v) { return v < uint64_t(kYClamp) ? int32_t(v) : kYClamp; }
 
-__device__ __forceinline__ void fill_tiles_ebwd(int L, int n, const int32_t *BC, const int32_t *Y,
+__device__ __forceinline__ void fill_tiles_ebwd(int L, int n, const int32_t *BC, const int32_t *NY,
                                                 const int32_t *prev, int32_t *best)
 {
     const int t = threadIdx.x, nt = blockDim.x;
@@ -303,18 +490,8 @@ __device__ __forceinline__ void fill_tiles_ebwd(int L, int n, const int32_t *BC,
     const int ng = (nb + 7) / 8;
     const int ntiles = 4 * ng * (ng + 1);
     for (int q = t; q < ntiles; q += nt) {
-        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
-        while (4 * (g + 1) * (g + 2) <= q) ++g;
-        while (g > 0 && 4 * g * (g + 1) > q) --g;
-        const int r = q - 4 * g * (g + 1);
-        const int b = 8 * g + r / (g + 1);
-        const int j = r % (g + 1);
-        if (b >= nb) continue;
-        const int bot = n + kRB * b;
-        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
-        const int k0 = n - 1 + kKC * j;
-        if (k0 > top - 1) continue;
-        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        int bot, top, k0, k1;
+        if (!decode_tile(q, L, n, nb, bot, top, k0, k1)) continue;
         int32_t R[kRB], acc[kRB];
 #pragma unroll
         for (int jj = 0; jj < kRB; ++jj) {
@@ -323,20 +500,28 @@ __device__ __forceinline__ void fill_tiles_ebwd(int L, int n, const int32_t *BC,
             acc[jj] = 0x7fffffff;
         }
         const int kf = k1 < bot ? k1 : bot;
-        for (int k = k0; k < kf; ++k) {
-            const int32_t v = prev[skew(k)], y = Y[skew(k)];
+        int k = k0;
+        for (; k + 1 < kf; k += 2) {
+            const int32_t v0 = prev[skew(k)], y0 = NY[skew(k)];
+            const int32_t v1 = prev[skew(k + 1)], y1 = NY[skew(k + 1)];
 #pragma unroll
-            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(v, R[jj] - y));
+            for (int jj = 0; jj < kRB; ++jj)
+                acc[jj] = __vimin3_s32(acc[jj], __viaddmax_s32(R[jj], y0, v0), __viaddmax_s32(R[jj], y1, v1));
+        }
+        if (k < kf) {
+            const int32_t v0 = prev[skew(k)], y0 = NY[skew(k)];
+#pragma unroll
+            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], __viaddmax_s32(R[jj], y0, v0));
         }
         if (k1 > bot) {
 #pragma unroll
             for (int u = 0; u < kRB - 1; ++u) {
-                const int k = bot + u;
-                if (k >= k1) break;
-                if (k < k0) continue;
-                const int32_t v = prev[skew(k)], y = Y[skew(k)];
+                const int kk = bot + u;
+                if (kk >= k1) break;
+                if (kk < k0) continue;
+                const int32_t v0 = prev[skew(kk)], y0 = NY[skew(kk)];
 #pragma unroll
-                for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(v, R[jj] - y));
+                for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = min(acc[jj], __viaddmax_s32(R[jj], y0, v0));
             }
         }
 #pragma unroll
@@ -350,14 +535,14 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
                            uint32_t *bitsw, int32_t *table)
 {
     const int L = a.L, t = threadIdx.x, nt = blockDim.x, Ls = group_ls(L);
-    // bytes [0, 8Ls): GTR (64-bit); then BCR, two columns, partial minima, Y (32-bit).
+    // bytes [0, 8Ls): GTR (64-bit); then BCR, two columns, partial minima, NY (32-bit).
     // P64c / P64x occupy bytes [16Ls, 32Ls): read before anything past 16Ls is written.
     uint64_t *GT = reinterpret_cast<uint64_t *>(arrays);
     int32_t *BC = reinterpret_cast<int32_t *>(arrays + size_t(8) * Ls);
     int32_t *colA = BC + Ls;
     int32_t *colB = colA + Ls;
     int32_t *best = colB + Ls;
-    int32_t *Y = best + Ls;
+    int32_t *NY = best + Ls;
     for (int m = t; m <= L; m += nt) {
         GT[skew(m)] = P64x[m];
         BC[skew(m)] = int32_t(P64c[m]);
@@ -369,12 +554,12 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
         colA[skew(m)] = v;
         best[skew(m)] = 0x7fffffff;
         table[tri_index(L, m, 1)] = v;
-        Y[skew(m)] = yclamp(dtv + GT[skew(m)]);
+        NY[skew(m)] = -yclamp(dtv + GT[skew(m)]);
     }
     __syncthreads();
     int32_t *prev = colA, *cur = colB;
     for (int n = 2; n <= L; ++n) {
-        fill_tiles_ebwd(L, n, BC, Y, prev, best);
+        fill_tiles_ebwd(L, n, BC, NY, prev, best);
         __syncthreads();
         const int64_t cbase = tri_col(L, n) - n;
         for (int m = n + t; m <= L; m += nt) {
@@ -383,7 +568,7 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
             best[skew(m)] = 0x7fffffff;
             table[cbase + m] = v;
         }
-        for (int k = n + t; k <= L; k += nt) Y[skew(k)] = yclamp(uint64_t(n) * dtv + GT[skew(k)]);
+        for (int k = n + t; k <= L; k += nt) NY[skew(k)] = -yclamp(uint64_t(n) * dtv + GT[skew(k)]);
         __syncthreads();
         int32_t *tmp = prev;
         prev = cur;
@@ -457,8 +642,9 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
 // A[k] and Q[m] are large but only a non-negative difference below 2^30 matters,
 // so inside a tile both are taken relative to P at the tile's lowest row: when
 // the tile's rows span less than 2^30 of transfer, A - P[bot] clamped below at
-// -2^30 and Q - P[bot] are signed 32-bit and the transition is subtract, max,
-// min; other tiles use the same formula in 64-bit. Candidates differ from Eq. 8's
+// -2^30 and Q - P[bot] are signed 32-bit and the transition is one add-then-max
+// (two candidates folding with one 3-input min); other tiles use the same
+// formula in 64-bit. Candidates differ from Eq. 8's
 // by the row constant n*dt + P[m] + G[m]: every argmin is unchanged, and
 // F[L][n] = E[L][n] + n*dt + P[L]. Needs FC[L] < 2^29.
 constexpr int32_t kSpan = 1 << 30;
@@ -472,48 +658,48 @@ __device__ __forceinline__ void fill_tiles_efwd(int L, int n, uint64_t dtv, cons
     const int ng = (nb + 7) / 8;
     const int ntiles = 4 * ng * (ng + 1);
     for (int q = t; q < ntiles; q += nt) {
-        int g = int((sqrtf(1.0f + float(q)) - 1.0f) * 0.5f);
-        while (4 * (g + 1) * (g + 2) <= q) ++g;
-        while (g > 0 && 4 * g * (g + 1) > q) --g;
-        const int r = q - 4 * g * (g + 1);
-        const int b = 8 * g + r / (g + 1);
-        const int j = r % (g + 1);
-        if (b >= nb) continue;
-        const int bot = n + kRB * b;
-        const int top = bot + kRB - 1 < L ? bot + kRB - 1 : L;
-        const int k0 = n - 1 + kKC * j;
-        if (k0 > top - 1) continue;
-        const int k1 = k0 + kKC < top ? k0 + kKC : top;  // exclusive
+        int bot, top, k0, k1;
+        if (!decode_tile(q, L, n, nb, bot, top, k0, k1)) continue;
         const int kf = k1 < bot ? k1 : bot;
         const uint64_t base = P[skew(bot)];
         int32_t acc[kRB];
 #pragma unroll
         for (int jj = 0; jj < kRB; ++jj) acc[jj] = 0x7fffffff;
         if (dtv + (P[skew(top)] - base) < uint64_t(kSpan)) {
-            int32_t Qr[kRB];
+            int32_t NQr[kRB];  // -(Q - base)
 #pragma unroll
             for (int jj = 0; jj < kRB; ++jj) {
                 const int m = bot + jj <= top ? bot + jj : top;
-                Qr[jj] = int32_t(dtv + (P[skew(m)] - base));
+                NQr[jj] = -int32_t(dtv + (P[skew(m)] - base));
             }
-            for (int k = k0; k < kf; ++k) {
+            auto rel = [&](int k) {  // A[k] - base, clamped below at -2^30
                 const int64_t ad = int64_t(A[skew(k)] - base);
-                const int32_t a = ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
-                const int32_t gk = G[skew(k)];
+                return ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
+            };
+            int k = k0;
+            for (; k + 1 < kf; k += 2) {
+                const int32_t a0 = rel(k), g0 = G[skew(k)];
+                const int32_t a1 = rel(k + 1), g1 = G[skew(k + 1)];
 #pragma unroll
-                for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(a - Qr[jj], gk));
+                for (int jj = 0; jj < kRB; ++jj)
+                    acc[jj] = __vimin3_s32(acc[jj], __viaddmax_s32(a0, NQr[jj], g0),
+                                           __viaddmax_s32(a1, NQr[jj], g1));
+            }
+            if (k < kf) {
+                const int32_t a0 = rel(k), g0 = G[skew(k)];
+#pragma unroll
+                for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], __viaddmax_s32(a0, NQr[jj], g0));
             }
             if (k1 > bot) {
 #pragma unroll
                 for (int u = 0; u < kRB - 1; ++u) {
-                    const int k = bot + u;
-                    if (k >= k1) break;
-                    if (k < k0) continue;
-                    const int64_t ad = int64_t(A[skew(k)] - base);
-                    const int32_t a = ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
-                    const int32_t gk = G[skew(k)];
+                    const int kk = bot + u;
+                    if (kk >= k1) break;
+                    if (kk < k0) continue;
+                    const int32_t a0 = rel(kk), g0 = G[skew(kk)];
 #pragma unroll
-                    for (int jj = u + 1; jj < kRB; ++jj) acc[jj] = min(acc[jj], max(a - Qr[jj], gk));
+                    for (int jj = u + 1; jj < kRB; ++jj)
+                        acc[jj] = min(acc[jj], __viaddmax_s32(a0, NQr[jj], g0));
                 }
             }
         } else {  // wide tile: the same candidates in 64-bit
@@ -689,7 +875,7 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
         const int any_neg = __syncthreads_or(bad_neg);
         const int any_big = __syncthreads_or(bad_big);
         int st = DC_OK;
-        bool narrow = false;
+        bool narrow = false, shifted32 = false;
         uint64_t shift = 0;
         if (any_neg) {
             st = DC_ERR_NEGATIVE;
@@ -711,7 +897,9 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
                 shift = sx - cx;
                 block_prefix_u64(P64c, L, scratch);
                 block_prefix_u64(P64x, L, scratch);
-                narrow = sc + cx + uint64_t(L) * uint64_t(dti) <= kNarrowLimit;
+                const uint64_t bound = sc + cx + uint64_t(L) * uint64_t(dti);
+                narrow = bound <= kNarrowLimit;
+                shifted32 = bound <= kShiftedLimit;
             }
         }
         if (st != DC_OK) {
@@ -724,15 +912,18 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
             __syncthreads();
             continue;
         }
-        if (narrow)
-            solve<uint32_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
-                                 reinterpret_cast<uint32_t *>(slot));
+        if (shifted32)
+            solve_s32<FWD>(a, i, dti, sx, P64c, P64x, arrays, bitsw,
+                           reinterpret_cast<int32_t *>(slot));
         else if (!FWD && sc < uint64_t(kYClamp))
             solve_ebwd(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                        reinterpret_cast<int32_t *>(slot));
         else if (FWD && sc < uint64_t(1) << 29)
             solve_efwd(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                        reinterpret_cast<int32_t *>(slot));
+        else if (narrow)
+            solve<uint32_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
+                                 reinterpret_cast<uint32_t *>(slot));
         else
             solve<uint64_t, FWD>(a, i, dti, shift, P64c, P64x, arrays, bitsw,
                                  reinterpret_cast<uint64_t *>(slot));

@@ -2,25 +2,36 @@
 // Eq. 9 / Algorithm 4), 32-bit arithmetic, runtime loops.
 //
 // Same processing-order template as the other kernels:
-//   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
+//   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c,
+// solved in the shifted form of the short-L kernel: values relative to the
+// start of the cell's last transfer, so that a transition is one 32-bit
+// add-then-max and the minimum runs on 3-input mins (1.5 integer-ALU
+// instructions per transition):
+//   forward : B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
+//   backward: E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),
+// with G[k] = FC[L] - FC[k], NQ[m] = -(dt + P[m]), NGT[k] = -(transfer prefix),
+// B[m][1] = FC[L], E[m][1] = BC[m]; the makespan is min_n (B or E)[L][n] + n*dt
+// plus the transfer sum. Every candidate differs from Eq. 8/9's by a constant of
+// its row, so every argmin is the same.
 //
 // Design (GB300):
-//  * one instance per thread; the lane's S, R and current column live in its
-//    slice of shared memory (lane-interleaved: value v at word 32*v + lane, so a
-//    warp's accesses never conflict);
+//  * one instance per thread; the lane's two per-layer arrays and its current
+//    column live in its slice of shared memory (lane-interleaved: value v at
+//    word 32*v + lane, so a warp's accesses never conflict);
 //  * register blocking: a column is filled in blocks of kB = 8 consecutive rows
-//    held in registers; every X[k][n-1], S[k] pair read from shared memory feeds
-//    kB transitions (max, subtract, min). Rows are visited top-down so that the
-//    column is updated in place: a block reads only rows below its own top,
-//    which still hold column n-1;
+//    held in registers; every two (column, array) pairs read from shared memory
+//    feed 2*kB transitions. Rows are visited top-down so that the column is
+//    updated in place: a block reads only rows below its own top, which still
+//    hold column n-1;
 //  * transfer costs capped at the total compute (exact, as in the short-L
-//    kernel), so that 32-bit values suffice for nearly every instance;
+//    kernel); the shifted values fit in signed 32 bits whenever the capped bound
+//    L*dt + sum(comp) + sum(capped xfer) is below 2^31;
 //  * value-only fill with deferred argmin, as in the short-L kernel: columns
 //    2..kKeep are written to a per-thread slot of the caller's workspace (L2
 //    resident, coalesced across the warp) and the traceback re-derives each
 //    Path[m][n] as the lowest k whose candidate equals the cell. Instances whose
-//    optimum needs a deeper column, or whose values need 64 bits, are put on a
-//    work list that the CTA-per-instance kernel solves afterwards;
+//    optimum needs a deeper column, or whose values need more than 31 bits, are
+//    put on a work list that the CTA-per-instance kernel solves afterwards;
 //  * persistent single-warp CTAs claim 32-instance tiles from an atomic ticket,
 //    so the long, uneven per-tile work balances across the GPU.
 #include "common.cuh"
@@ -55,8 +66,8 @@ __global__ void __launch_bounds__(32)
     extern __shared__ uint32_t smem[];
     const int lane = threadIdx.x;
     const int W = words_for(L);
-    uint32_t *lw = smem + lane;  // S at v in [0, L], R at [L+1, 2L+1], col at [2L+2, 3L+2]
-    const int oR = L + 1, oC = 2 * (L + 1);
+    uint32_t *lw = smem + lane;  // U at v in [0, L], V at [L+1, 2L+1], column at [2L+2, 3L+2]
+    const int oV = L + 1, oC = 2 * (L + 1);
     const int64_t slot = int64_t(blockIdx.x) * 32 + lane;
     uint32_t *myslot = tb + slot;  // cell c at myslot[c * nslots]
     const int keep = mid_keep_last(L);
@@ -92,72 +103,87 @@ __global__ void __launch_bounds__(32)
             for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
             continue;
         }
+        // per-layer arrays (U, V) = (NQ, G) forward, (BC, NGT) backward, written
+        // with wrapping 32-bit arithmetic: used only when the range check passes
         uint64_t pc = 0, pxc = 0;
-        lw[0] = 0u;
-        lw[32 * oR] = 0u;
+        const uint32_t dtu = uint32_t(dti), tcu = uint32_t(tc);
+        lw[0] = FWD ? 0u - dtu : 0u;
+        lw[32 * oV] = FWD ? tcu : 0u;
         for (int r = 1; r <= L; ++r) {
             const int col = FWD ? r - 1 : L - r;
             const uint64_t cv = uint64_t(__ldg(crow + col)), xv = uint64_t(__ldg(xrow + col));
             pc += cv;
             pxc += xv < tc ? xv : tc;
-            lw[32 * r] = uint32_t(FWD ? pc : pxc);         // S
-            lw[32 * (oR + r)] = uint32_t(FWD ? pxc : pc);  // R base
+            lw[32 * r] = FWD ? 0u - dtu - uint32_t(pxc) : uint32_t(pc);
+            lw[32 * (oV + r)] = FWD ? tcu - uint32_t(pc) : 0u - uint32_t(pxc);
         }
-        const uint64_t shift = px - pxc;
-        if (pc + pxc + uint64_t(L) * uint64_t(dti) > kNarrowLimit) {
+        if (pc + pxc + uint64_t(L) * uint64_t(dti) > kShiftedLimit) {
             list[atomicAdd(list_count, 1u)] = uint32_t(i);
             continue;
         }
+        const int32_t *U = reinterpret_cast<const int32_t *>(lw);
+        const int32_t *V = U + 32 * oV;
+        int32_t *C = reinterpret_cast<int32_t *>(lw) + 32 * oC;
 
         // ---- fill
-        const uint32_t dtv = uint32_t(dti);
-        const uint32_t c = FWD ? 0u : dtv;
-        for (int m = 1; m <= L; ++m) {
-            const uint32_t rb = lw[32 * (oR + m)];
-            lw[32 * (oC + m)] = (FWD ? dtv + rb : rb) + lw[32 * m] + c;
-        }
-        uint32_t Tbest = lw[32 * (oC + L)];
+        const int32_t dt32 = int32_t(dti), fcL = int32_t(tc);
+        for (int m = 1; m <= L; ++m) C[32 * m] = FWD ? fcL - U[32 * m] - dt32 : U[32 * m];
+        int32_t bestV = (FWD ? fcL : U[32 * L]) + dt32;
         int s = 1;
         for (int n = 2; n <= L; ++n) {
-            const uint32_t ndt = uint32_t(n) * dtv;
+            const int32_t ndt1 = (n - 1) * dt32;
+            int32_t last = 0;
             for (int top = L; top >= n; top -= kB) {
                 const int bot = top - kB + 1 > n ? top - kB + 1 : n;
-                uint32_t R[kB], best[kB];
+                int32_t Ur[kB], best[kB];
 #pragma unroll
                 for (int j = 0; j < kB; ++j) {
                     const int m = bot + j <= top ? bot + j : top;
-                    const uint32_t rb = lw[32 * (oR + m)];
-                    R[j] = FWD ? ndt + rb : rb;
-                    best[j] = 0xffffffffu;
+                    Ur[j] = FWD ? U[32 * m] : U[32 * m] - ndt1;
+                    best[j] = 0x7fffffff;
                 }
-                // k below the block: every row of the block takes it
-                for (int k = n - 1; k < bot; ++k) {
-                    const uint32_t v = lw[32 * (oC + k)], sk = lw[32 * k];
+                // k below the block, two at a time: every row of the block takes them
+                int k = n - 1;
+                for (; k + 1 < bot; k += 2) {
+                    const int32_t c0 = C[32 * k], v0 = V[32 * k];
+                    const int32_t c1 = C[32 * (k + 1)], v1 = V[32 * (k + 1)];
 #pragma unroll
-                    for (int j = 0; j < kB; ++j) best[j] = dmin(best[j], dmax(v, R[j]) - sk);
+                    for (int j = 0; j < kB; ++j) {
+                        const int32_t x0 = FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0);
+                        const int32_t x1 = FWD ? __viaddmax_s32(c1, Ur[j], v1) : __viaddmax_s32(Ur[j], v1, c1);
+                        best[j] = __vimin3_s32(best[j], x0, x1);
+                    }
+                }
+                if (k < bot) {
+                    const int32_t c0 = C[32 * k], v0 = V[32 * k];
+#pragma unroll
+                    for (int j = 0; j < kB; ++j)
+                        best[j] = min(best[j], FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0));
                 }
                 // k inside the block: row bot+j takes k < bot+j
 #pragma unroll
                 for (int t = 0; t < kB - 1; ++t) {
-                    const int k = bot + t;
-                    if (k >= top) break;
-                    const uint32_t v = lw[32 * (oC + k)], sk = lw[32 * k];
+                    const int kk = bot + t;
+                    if (kk >= top) break;
+                    const int32_t c0 = C[32 * kk], v0 = V[32 * kk];
 #pragma unroll
-                    for (int j = t + 1; j < kB; ++j) best[j] = dmin(best[j], dmax(v, R[j]) - sk);
+                    for (int j = t + 1; j < kB; ++j)
+                        best[j] = min(best[j], FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0));
                 }
 #pragma unroll
                 for (int j = 0; j < kB; ++j) {
                     const int m = bot + j;
                     if (m <= top) {
-                        const uint32_t val = best[j] + lw[32 * m] + c;
-                        lw[32 * (oC + m)] = val;
-                        if (n <= keep) myslot[int64_t(mid_cell(L, m, n)) * nslots] = val;
+                        if (m == L) last = best[j];
+                        const int32_t val = FWD ? best[j] - U[32 * m] - dt32 : best[j];
+                        C[32 * m] = val;
+                        if (n <= keep) myslot[int64_t(mid_cell(L, m, n)) * nslots] = uint32_t(val);
                     }
                 }
             }
-            const uint32_t last = lw[32 * (oC + L)];
-            if (last < Tbest) {  // strict: the lowest n wins ties
-                Tbest = last;
+            const int32_t v = last + n * dt32;
+            if (v < bestV) {  // strict: the lowest n wins ties
+                bestV = v;
                 s = n;
             }
         }
@@ -169,30 +195,28 @@ __global__ void __launch_bounds__(32)
         // ---- traceback: lowest k whose candidate equals the cell
         uint32_t word0 = 0u, word1 = 0u;  // L <= 64: W <= 2
         int err = 0, m = L, n = s;
-        uint32_t cell = Tbest;
+        int32_t target = bestV - s * dt32;  // B[L][s] or E[L][s]
         while (n > 1) {
-            const uint32_t rm = lw[32 * (oR + m)];
-            const uint32_t R = FWD ? uint32_t(n) * dtv + rm : rm;
-            const uint32_t target = cell - lw[32 * m] - c;
+            const int32_t um = U[32 * m];
+            const int32_t Rn = um - (n - 1) * dt32;  // backward only
             // candidates in groups of 4 (loads issued together, lowest match wins)
             int k = -1;
-            uint32_t fk = 0;
+            int32_t fk = 0;
             for (int k0 = n - 1; k0 < m && k < 0; k0 += 4) {
-                uint32_t f[4], sk[4];
+                int32_t f[4], v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
-                    if (n - 1 == 1) {
-                        const uint32_t rb = lw[32 * (oR + kk)];
-                        f[u] = (FWD ? dtv + rb : rb) + lw[32 * kk] + c;
-                    } else {
-                        f[u] = myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots];
-                    }
-                    sk[u] = lw[32 * kk];
+                    v[u] = V[32 * kk];
+                    if (n - 1 == 1)  // column 1 is not stored
+                        f[u] = FWD ? fcL - U[32 * kk] - dt32 : U[32 * kk];
+                    else
+                        f[u] = int32_t(myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots]);
                 }
 #pragma unroll
                 for (int u = 3; u >= 0; --u) {
-                    if (k0 + u < m && dmax(f[u], R) - sk[u] == target) {
+                    const int32_t cand = FWD ? __viaddmax_s32(f[u], um, v[u]) : __viaddmax_s32(Rn, v[u], f[u]);
+                    if (k0 + u < m && cand == target) {
                         k = k0 + u;
                         fk = f[u];
                     }
@@ -206,11 +230,11 @@ __global__ void __launch_bounds__(32)
                 word0 |= 1u << (k - 1);
             else
                 word1 |= 1u << (k - 33);
+            target = FWD ? fk + U[32 * k] + dt32 : fk;  // B[k][n-1] = A + P[k]
             m = k;
             n -= 1;
-            cell = fk;
         }
-        makespan[i] = int64_t(uint64_t(Tbest) + shift);
+        makespan[i] = int64_t(uint64_t(uint32_t(bestV)) + px);
         if (nseg) nseg[i] = s;
         if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
         bits[i * W] = word0;

@@ -207,6 +207,160 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
     return true;
 }
 
+// ---------------------------------------------------------------------------
+// The 32-bit pass in shifted form. Every value is taken relative to the time
+// the last pull (forward) or push (backward) of its cell can start, which turns
+// a transition into one add-then-max and the minimum into 3-input mins: on
+// GB300 both are single integer-ALU instructions (the DPX forms), so a transition
+// costs 1.5 ALU-pipe instructions instead of 2.
+//
+// forward (P = transfer prefix, FC = compute prefix, G[k] = FC[L] - FC[k],
+// NQ[m] = -(dt + P[m])): with B = X - n*dt - P[m] + G[m] (X as above),
+//   B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
+//   B[m][1] = FC[L],  X[L][n] = B[L][n] + n*dt + P[L];
+// backward (BC = compute prefix, NGT[k] = -(transfer prefix)): with
+// E = X - n*dt - S[m],
+//   E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),  E[m][1] = BC[m],
+//   X[L][n] = E[L][n] + n*dt + S[L].
+// Each candidate differs from Eq. 8/9's by a constant of its row, so every
+// argmin is the same. All values and sums lie in [-2^31, 2^31) when the capped
+// bound L*dt + sum(comp) + sum(capped xfer) is below 2^31; other instances take
+// the 64-bit pass. The table stores A (forward) or E (backward) for columns
+// 2..kKeepCols; the lane's two arrays hold NQ and G (forward) or BC and NGT.
+
+// Minimum of c[0..cnt-1] (cnt a compile-time constant after unrolling): two
+// chains of 3-input mins, so that each row has two independent dependency chains
+// and the rows of a column interleave.
+template <int N>
+__device__ __forceinline__ int32_t min_fold3(const int32_t (&c)[N], int cnt)
+{
+    if (cnt == 1) return c[0];
+    if (cnt == 2) return min(c[0], c[1]);
+    int32_t a = c[0], b = c[1];
+    int j = 2;
+#pragma unroll
+    for (; j + 3 < cnt; j += 4) {
+        a = __vimin3_s32(a, c[j], c[j + 1]);
+        b = __vimin3_s32(b, c[j + 2], c[j + 3]);
+    }
+    if (j + 1 < cnt) return __vimin3_s32(__vimin3_s32(a, b, c[j]), c[j + 1], cnt > j + 2 ? c[j + 2] : c[j + 1]);
+    if (j < cnt) return __vimin3_s32(a, b, c[j]);
+    return min(a, b);
+}
+
+template <int L, bool FWD>
+__device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
+                                       int32_t dt, int32_t fcL, int32_t *lw, int32_t &bestV,
+                                       int &best_s)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    // forward: U = NQ, V = G, col = A; backward: U = BC, V = NGT, col = E
+    int32_t col[L + 1];
+#pragma unroll
+    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL - U[m] - dt : U[m];
+    bestV = (FWD ? fcL : U[L]) + dt;
+    best_s = 1;
+#pragma unroll
+    for (int n = 2; n <= L; ++n) {
+        int32_t last = 0;  // B[L][n] or E[L][n]
+#pragma unroll
+        for (int m = L; m >= n; --m) {  // descending: column n overwrites column n-1 in place
+            const int cnt = m - n + 1;  // k = n-1 .. m-1
+            int32_t c[L];
+            if (FWD) {
+#pragma unroll
+                for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(col[n - 1 + j], U[m], V[n - 1 + j]);
+            } else {
+                const int32_t Rn = U[m] - (n - 1) * dt;
+#pragma unroll
+                for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(Rn, V[n - 1 + j], col[n - 1 + j]);
+            }
+            const int32_t b = min_fold3<L>(c, cnt);
+            if (m == L) last = b;
+            col[m] = FWD ? b - U[m] - dt : b;
+            if (n <= K::kLast) lw[32 * cell2(L, m, n)] = col[m];
+        }
+        const int32_t v = last + n * dt;
+        if (v < bestV) {  // strict: the lowest n wins ties
+            bestV = v;
+            best_s = n;
+        }
+    }
+}
+
+// The fill, the traceback and the outputs of one instance in shifted form.
+// Returns false (writing nothing) when the traceback needs a column the pass did
+// not keep.
+template <int L, bool FWD>
+__device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+                                        int64_t dti, uint64_t xraw, int32_t *lw, int64_t i,
+                                        int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                                        int32_t *status)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    constexpr int W = (L - 1 + 31) / 32;
+    const int32_t dt = int32_t(dti);
+    const int32_t fcL = int32_t(Pc[L]);
+    int32_t U[L + 1], V[L + 1];
+#pragma unroll
+    for (int m = 0; m <= L; ++m) {
+        U[m] = FWD ? -(dt + int32_t(Px[m])) : int32_t(Pc[m]);
+        V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
+        lw[32 * (K::kOffR + m)] = U[m];
+        lw[32 * (K::kOffS + m)] = V[m];
+    }
+    int32_t bestV;
+    int s;
+    fill_e<L, FWD>(U, V, dt, fcL, lw, bestV, s);
+    if (s - 1 > K::kLast && s - 1 >= 2) return false;
+
+    // from (L, s) step to the lowest k whose candidate equals the cell, set
+    // p_k / g_k, continue at (k, n-1)
+    uint32_t word = 0;
+    int err = 0;
+    int m = L, n = s;
+    int32_t target = bestV - s * dt;  // B[L][s] or E[L][s]
+    while (n > 1) {
+        const int32_t um = lds(lw, K::kOffR + m);
+        const int32_t Rn = um - (n - 1) * dt;  // backward only
+        int k = -1;
+        int32_t fk = 0;
+        for (int k0 = n - 1; k0 < m && k < 0; k0 += kTbGroup) {
+            int32_t f[kTbGroup], v[kTbGroup];
+#pragma unroll
+            for (int u = 0; u < kTbGroup; ++u) {
+                const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
+                v[u] = lds(lw, K::kOffS + kk);
+                if (n - 1 == 1)  // column 1 is not stored
+                    f[u] = FWD ? fcL - lds(lw, K::kOffR + kk) - dt : lds(lw, K::kOffR + kk);
+                else
+                    f[u] = lds(lw, cell2(L, kk, n - 1));
+            }
+#pragma unroll
+            for (int u = kTbGroup - 1; u >= 0; --u) {
+                const int32_t cand = FWD ? __viaddmax_s32(f[u], um, v[u]) : __viaddmax_s32(Rn, v[u], f[u]);
+                if (k0 + u < m && cand == target) {
+                    k = k0 + u;
+                    fk = f[u];
+                }
+            }
+        }
+        if (k < 0) {  // cannot happen: the fill and this check use the same arithmetic
+            err = 1;
+            break;
+        }
+        word |= 1u << ((k - 1) & 31);
+        target = FWD ? fk + lds(lw, K::kOffR + k) + dt : fk;  // B[k][n-1] = A + P[k]
+        m = k;
+        n -= 1;
+    }
+    makespan[i] = int64_t(uint64_t(uint32_t(bestV)) + xraw);
+    if (nseg) nseg[i] = s;
+    if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+    if (W > 0) bits[i * W] = word;
+    return true;
+}
+
 __device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
 {
     const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
@@ -288,7 +442,7 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
     const int lane = threadIdx.x;
     int64_t *stC = reinterpret_cast<int64_t *>(smem);
     int64_t *stX = stC + 32 * K::kStride;
-    uint32_t *lw = reinterpret_cast<uint32_t *>(smem) + lane;
+    int32_t *lw = reinterpret_cast<int32_t *>(smem) + lane;
 
     const int64_t tiles = (batch + 31) / 32;
     int64_t tile = blockIdx.x;
@@ -322,9 +476,8 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         const uint64_t bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];  // capped
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
-        } else if (bound > kNarrowLimit ||
-                   !solve<L, FWD, uint32_t, kKeepCols>(Pc, Px, dti, xraw - Px[L], lw, i,
-                                                       makespan, bits, nseg, status)) {
+        } else if (bound > kShiftedLimit ||
+                   !solve_e<L, FWD>(Pc, Px, dti, xraw, lw, i, makespan, bits, nseg, status)) {
             // 64-bit values, or a traceback deeper than the kept columns: work list
             wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
         }
