@@ -16,11 +16,14 @@
 //
 // Design (GB300):
 //  * one instance per thread; the lane's two per-layer arrays and its current
-//    column live in its slice of shared memory (lane-interleaved: value v at
-//    word 32*v + lane, so a warp's accesses never conflict);
+//    column live in its slice of shared memory, lane-interleaved so that a
+//    warp's accesses never conflict (U[v] at word 32*v + lane; the column and V
+//    as 64-bit pairs at 32*v + lane, one load per candidate k);
 //  * register blocking: a column is filled in blocks of kB = 8 consecutive rows
-//    held in registers; every two (column, array) pairs read from shared memory
-//    feed 2*kB transitions. Rows are visited top-down so that the column is
+//    held in registers; every (column, V) pair read from shared memory feeds kB
+//    transitions. A full block's own triangle (row bot+j takes k < bot+j) is
+//    unrolled without branches; only a column's lowest, partial block takes the
+//    general path. Rows are visited top-down so that the column is
 //    updated in place: a block reads only rows below its own top, which still
 //    hold column n-1;
 //  * transfer costs capped at the total compute (exact, as in the short-L
@@ -39,7 +42,7 @@
 namespace dc {
 namespace {
 
-constexpr int kB = 8;      // rows per register block
+constexpr int kB = 8;  // rows per register block
 constexpr int kKeep = 8;  // last column kept for the traceback
 
 __host__ __device__ inline int mid_keep_last(int L) { return L - 1 < kKeep ? L - 1 : kKeep; }
@@ -66,8 +69,10 @@ __global__ void __launch_bounds__(32)
     extern __shared__ uint32_t smem[];
     const int lane = threadIdx.x;
     const int W = words_for(L);
-    uint32_t *lw = smem + lane;  // U at v in [0, L], V at [L+1, 2L+1], column at [2L+2, 3L+2]
-    const int oV = L + 1, oC = 2 * (L + 1);
+    // lane slices: U[v] at word 32*v + lane (v in [0, L]), then the current column
+    // and V as (C[v], V[v]) pairs at 64-bit word 32*v + lane
+    uint32_t *lw = smem + lane;
+    int2 *pv = reinterpret_cast<int2 *>(smem + 32 * (L + 1)) + lane;
     const int64_t slot = int64_t(blockIdx.x) * 32 + lane;
     uint32_t *myslot = tb + slot;  // cell c at myslot[c * nslots]
     const int keep = mid_keep_last(L);
@@ -108,26 +113,24 @@ __global__ void __launch_bounds__(32)
         uint64_t pc = 0, pxc = 0;
         const uint32_t dtu = uint32_t(dti), tcu = uint32_t(tc);
         lw[0] = FWD ? 0u - dtu : 0u;
-        lw[32 * oV] = FWD ? tcu : 0u;
+        pv[0].y = FWD ? int32_t(tcu) : 0;
         for (int r = 1; r <= L; ++r) {
             const int col = FWD ? r - 1 : L - r;
             const uint64_t cv = uint64_t(__ldg(crow + col)), xv = uint64_t(__ldg(xrow + col));
             pc += cv;
             pxc += xv < tc ? xv : tc;
             lw[32 * r] = FWD ? 0u - dtu - uint32_t(pxc) : uint32_t(pc);
-            lw[32 * (oV + r)] = FWD ? tcu - uint32_t(pc) : 0u - uint32_t(pxc);
+            pv[32 * r].y = int32_t(FWD ? tcu - uint32_t(pc) : 0u - uint32_t(pxc));
         }
         if (pc + pxc + uint64_t(L) * uint64_t(dti) > kShiftedLimit) {
             list[atomicAdd(list_count, 1u)] = uint32_t(i);
             continue;
         }
         const int32_t *U = reinterpret_cast<const int32_t *>(lw);
-        const int32_t *V = U + 32 * oV;
-        int32_t *C = reinterpret_cast<int32_t *>(lw) + 32 * oC;
 
         // ---- fill
         const int32_t dt32 = int32_t(dti), fcL = int32_t(tc);
-        for (int m = 1; m <= L; ++m) C[32 * m] = FWD ? fcL - U[32 * m] - dt32 : U[32 * m];
+        for (int m = 1; m <= L; ++m) pv[32 * m].x = FWD ? fcL - U[32 * m] - dt32 : U[32 * m];
         int32_t bestV = (FWD ? fcL : U[32 * L]) + dt32;
         int s = 1;
         for (int n = 2; n <= L; ++n) {
@@ -142,33 +145,63 @@ __global__ void __launch_bounds__(32)
                     Ur[j] = FWD ? U[32 * m] : U[32 * m] - ndt1;
                     best[j] = 0x7fffffff;
                 }
-                // k below the block, two at a time: every row of the block takes them
+                // k below the block, four then two at a time: every row of the
+                // block takes them; one 64-bit load brings a (column, V) pair
+                auto cand = [&](int2 p, int j) {
+                    return FWD ? __viaddmax_s32(p.x, Ur[j], p.y) : __viaddmax_s32(Ur[j], p.y, p.x);
+                };
                 int k = n - 1;
-                for (; k + 1 < bot; k += 2) {
-                    const int32_t c0 = C[32 * k], v0 = V[32 * k];
-                    const int32_t c1 = C[32 * (k + 1)], v1 = V[32 * (k + 1)];
+                for (; k + 3 < bot; k += 4) {
+                    const int2 p0 = pv[32 * k], p1 = pv[32 * (k + 1)];
+                    const int2 p2 = pv[32 * (k + 2)], p3 = pv[32 * (k + 3)];
 #pragma unroll
                     for (int j = 0; j < kB; ++j) {
-                        const int32_t x0 = FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0);
-                        const int32_t x1 = FWD ? __viaddmax_s32(c1, Ur[j], v1) : __viaddmax_s32(Ur[j], v1, c1);
-                        best[j] = __vimin3_s32(best[j], x0, x1);
+                        best[j] = __vimin3_s32(best[j], cand(p0, j), cand(p1, j));
+                        best[j] = __vimin3_s32(best[j], cand(p2, j), cand(p3, j));
                     }
                 }
-                if (k < bot) {
-                    const int32_t c0 = C[32 * k], v0 = V[32 * k];
+                if (k + 1 < bot) {
+                    const int2 p0 = pv[32 * k], p1 = pv[32 * (k + 1)];
 #pragma unroll
-                    for (int j = 0; j < kB; ++j)
-                        best[j] = min(best[j], FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0));
+                    for (int j = 0; j < kB; ++j) best[j] = __vimin3_s32(best[j], cand(p0, j), cand(p1, j));
+                    k += 2;
                 }
-                // k inside the block: row bot+j takes k < bot+j
+                if (k < bot) {
+                    const int2 p0 = pv[32 * k];
+#pragma unroll
+                    for (int j = 0; j < kB; ++j) best[j] = min(best[j], cand(p0, j));
+                }
+                if (top - bot == kB - 1) {
+                    // full block, k inside it: row bot+j takes k = bot .. bot+j-1,
+                    // unrolled without branches, candidates paired into 3-input mins
+                    int2 q[kB - 1];
+#pragma unroll
+                    for (int t = 0; t < kB - 1; ++t) q[t] = pv[32 * (bot + t)];
+#pragma unroll
+                    for (int j = 1; j < kB; ++j) {
+                        int t = 0;
+#pragma unroll
+                        for (; t + 1 < j; t += 2) best[j] = __vimin3_s32(best[j], cand(q[t], j), cand(q[t + 1], j));
+                        if (t < j) best[j] = min(best[j], cand(q[t], j));
+                    }
+                    if (top == L) last = best[kB - 1];
+                    const int64_t cb = int64_t(mid_cell(L, bot, n)) * nslots;
+#pragma unroll
+                    for (int j = 0; j < kB; ++j) {
+                        const int32_t val = FWD ? best[j] - Ur[j] - dt32 : best[j];
+                        pv[32 * (bot + j)].x = val;
+                        if (n <= keep) myslot[cb + int64_t(j) * nslots] = uint32_t(val);
+                    }
+                    continue;
+                }
+                // partial block (the column's lowest), k inside it
 #pragma unroll
                 for (int t = 0; t < kB - 1; ++t) {
                     const int kk = bot + t;
                     if (kk >= top) break;
-                    const int32_t c0 = C[32 * kk], v0 = V[32 * kk];
+                    const int2 p0 = pv[32 * kk];
 #pragma unroll
-                    for (int j = t + 1; j < kB; ++j)
-                        best[j] = min(best[j], FWD ? __viaddmax_s32(c0, Ur[j], v0) : __viaddmax_s32(Ur[j], v0, c0));
+                    for (int j = t + 1; j < kB; ++j) best[j] = min(best[j], cand(p0, j));
                 }
 #pragma unroll
                 for (int j = 0; j < kB; ++j) {
@@ -176,7 +209,7 @@ __global__ void __launch_bounds__(32)
                     if (m <= top) {
                         if (m == L) last = best[j];
                         const int32_t val = FWD ? best[j] - U[32 * m] - dt32 : best[j];
-                        C[32 * m] = val;
+                        pv[32 * m].x = val;
                         if (n <= keep) myslot[int64_t(mid_cell(L, m, n)) * nslots] = uint32_t(val);
                     }
                 }
@@ -207,7 +240,7 @@ __global__ void __launch_bounds__(32)
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
-                    v[u] = V[32 * kk];
+                    v[u] = pv[32 * kk].y;
                     if (n - 1 == 1)  // column 1 is not stored
                         f[u] = FWD ? fcL - U[32 * kk] - dt32 : U[32 * kk];
                     else
