@@ -36,6 +36,11 @@ UNIT = "instances/s"
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_PATH = os.path.join(ROOT, "profiles", "dp_traffic.json")
 
+# Integer-ALU roof: GB300's maximum SM clock, and the instructions one
+# transition of the 32-bit passes takes (one add-then-max, half a 3-input min).
+MAX_SM_MHZ = 2070
+ALU_OPS_PER_TRANSITION = 1.5
+
 # Oracle sample sizes for the CPU baseline (instances per timed pass).
 CPU_SAMPLE = {"tiny": 4096, "alexnet": 1_000_000, "vgg16": 1_000_000, "resnet50": 65_536,
               "deepchain": 16}
@@ -130,6 +135,25 @@ def dp_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+# ------------------------------------------------------------ multi-rank
+def rank_config(base: dict, rank: int) -> dict:
+    """Weak scaling: each rank solves its own `batch` distinct instances; rank r
+    takes instance numbers [r*batch, (r+1)*batch) of the seeded stream (the
+    generator is counter-based, so the shards together are the world-size batch)."""
+    return wl.with_batch(base, base["batch"], inst0=base.get("inst0", 0) + rank * base["batch"])
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    """The slowest rank's value (a single process returns x)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ------------------------------------------------------------- reference arm
 def oracle_pass(cfg, sample: int, nthreads: int):
     """The oracle, as it stands, over the first `sample` instances of cfg:
@@ -200,7 +224,7 @@ def run_ours(args):
     if args.batch:
         base = wl.with_batch(base, args.batch)
     B, L = base["batch"], base["L"]
-    cfg = wl.with_batch(base, B, inst0=rank * B)  # distinct instances per rank
+    cfg = rank_config(base, rank)  # distinct instances per rank
     W = dc.words(L)
 
     prof = {k: torch.empty((B, L), dtype=torch.int64, device=dev) for k in ("fc", "pt", "bc", "gt")}
@@ -257,10 +281,7 @@ def run_ours(args):
     ms = start.elapsed_time(end) / max(args.steps, 1)
     seg = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])
     gen_ms, fwd_ms, bwd_ms, eval_ms = seg.mean(axis=0)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dev)
 
     # ---- ALU roof: the DP's transition op mix, register-only, all SMs
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -301,15 +322,19 @@ def run_ours(args):
     trans = 2 * transitions(L) * B
     dp_s = (fwd_ms + bwd_ms) * 1e-3
     achieved = trans / dp_s / 1e9
-    peak = roof[0] / 1e9
+    # ALU roof from unit counts: 4 x 16 integer-ALU lanes per SM per clock, the
+    # 32-bit passes spend 1.5 ALU instructions per transition
+    peak = sms * 64 * MAX_SM_MHZ * 1e6 / ALU_OPS_PER_TRANSITION / 1e9
     traffic = None
     tr = load_json(TRAFFIC_PATH)
     if tr and tr.get("workload") == args.workload and tr.get("source_hash") == dp_source_hash():
         traffic = tr.get("bytes_per_launch")
     hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
     dp_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
-    small = L <= 16
-    launches_per_step = 1 + 2 * (2 if small else 1) + 2
+    # kernels of this library per step: the generator; per direction the 32-bit
+    # pass and the pass over its work list (L <= 64) or the per-instance kernel
+    # alone (L > 64); the two timeline replays
+    launches_per_step = 1 + 2 * (2 if L <= 64 else 1) + 2
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -327,9 +352,12 @@ def run_ours(args):
         "roofline": {"bound": "alu", "kernel": "dp_schedule (forward + backward)",
                      "achieved": achieved, "peak": peak, "unit": "Gtransitions/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "peak_source": "register-only probe of the same op mix (32-bit), "
-                                    f"{sms} SMs, measured in this run",
-                     "peak_u64": roof[1] / 1e9,
+                     "peak_source": f"{sms} SMs x 64 integer-ALU lanes x {MAX_SM_MHZ} MHz / "
+                                    f"{ALU_OPS_PER_TRANSITION} ALU instructions per transition",
+                     "peak_probe": roof[0] / 1e9,
+                     "peak_probe_source": "register-only loop of the 32-bit passes' op mix, "
+                                          "all SMs, measured in this run",
+                     "peak_u64_probe": roof[1] / 1e9,
                      "hbm": {"achieved_gbs": dp_gbs, "peak_gbs": hbm_peak,
                              "frac": dp_gbs / hbm_peak,
                              "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}},
@@ -379,12 +407,7 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     t1.record()
     torch.cuda.synchronize()
     barrier()
-    ms = t0.elapsed_time(t1) / steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t0.elapsed_time(t1) / steps, dev)
     return {"value": B * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps,
             "path": f"pinned host profiles -> dynacomm.HostPipeline ({pipe.chunks} chunks, "
