@@ -295,18 +295,17 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
 // the shifted form of the thread-per-instance kernels, all in signed 32 bits,
 // where a transition is one add-then-max and two candidates fold with one
 // 3-input min (1.5 integer-ALU instructions per transition):
-//   forward : B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
+//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k] - dt,
 //   backward: E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),
-// with G[k] = FC[L] - FC[k], NQ[m] = -(dt + P[m]) (P = transfer prefix),
-// NGT[k] = -(transfer prefix), B[m][1] = FC[L], E[m][1] = BC[m]; U = (NQ, BC) and
-// V = (G, NGT) per direction. The makespan is min_n (B or E)[L][n] + n*dt plus
+// with G[k] = FC[L] - FC[k], Q[m] = dt + P[m] (P = transfer prefix),
+// NGT[k] = -(transfer prefix), A[m][1] = FC[L] + P[m], E[m][1] = BC[m]; U = (Q, BC)
+// and V = (G, NGT) per direction, and both are min_k max(u[m] + V[k], C[k]). The makespan is min_n (B or E)[L][n] + n*dt plus
 // the transfer sum. Each candidate differs from Eq. 8/9's by a constant of its
 // row, so every argmin is unchanged. The table holds A (forward) or E.
 
-template <bool FWD>
 __device__ __forceinline__ int32_t cand_s32(int32_t col, int32_t u, int32_t v)
 {
-    return FWD ? __viaddmax_s32(col, u, v) : __viaddmax_s32(u, v, col);
+    return __viaddmax_s32(u, v, col);
 }
 
 template <bool FWD>
@@ -335,13 +334,13 @@ __device__ __forceinline__ void fill_tiles_s32(int L, int n, int32_t ndt1, const
             const int32_t c1 = prev[skew(k + 1)], v1 = V[skew(k + 1)];
 #pragma unroll
             for (int jj = 0; jj < kRB; ++jj)
-                acc[jj] = __vimin3_s32(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0),
-                                       cand_s32<FWD>(c1, Ur[jj], v1));
+                acc[jj] = __vimin3_s32(acc[jj], cand_s32(c0, Ur[jj], v0),
+                                       cand_s32(c1, Ur[jj], v1));
         }
         if (k < kf) {
             const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
 #pragma unroll
-            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0));
+            for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], cand_s32(c0, Ur[jj], v0));
         }
         if (k1 > bot) {  // row bot+jj takes k < bot+jj
 #pragma unroll
@@ -352,7 +351,7 @@ __device__ __forceinline__ void fill_tiles_s32(int L, int n, int32_t ndt1, const
                 const int32_t c0 = prev[skew(kk)], v0 = V[skew(kk)];
 #pragma unroll
                 for (int jj = u + 1; jj < kRB; ++jj)
-                    acc[jj] = min(acc[jj], cand_s32<FWD>(c0, Ur[jj], v0));
+                    acc[jj] = min(acc[jj], cand_s32(c0, Ur[jj], v0));
             }
         }
 #pragma unroll
@@ -377,12 +376,12 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
     const int32_t dt = int32_t(dti);
     const int32_t fcL = int32_t(P64c[L]);
     for (int m = t; m <= L; m += nt) {
-        U[skew(m)] = FWD ? -(dt + int32_t(P64x[m])) : int32_t(P64c[m]);
+        U[skew(m)] = FWD ? dt + int32_t(P64x[m]) : int32_t(P64c[m]);
         V[skew(m)] = FWD ? fcL - int32_t(P64c[m]) : -int32_t(P64x[m]);
     }
     __syncthreads();
     for (int m = 1 + t; m <= L; m += nt) {  // column 1
-        const int32_t v = FWD ? fcL - U[skew(m)] - dt : U[skew(m)];
+        const int32_t v = FWD ? fcL + U[skew(m)] - dt : U[skew(m)];
         colA[skew(m)] = v;
         best[skew(m)] = 0x7fffffff;
         table[tri_index(L, m, 1)] = v;
@@ -395,7 +394,7 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
         const int64_t cbase = tri_col(L, n) - n;
         for (int m = n + t; m <= L; m += nt) {
             const int32_t b = best[skew(m)];
-            const int32_t v = FWD ? b - U[skew(m)] - dt : b;
+            const int32_t v = FWD ? b - dt : b;
             cur[skew(m)] = v;
             best[skew(m)] = 0x7fffffff;
             table[cbase + m] = v;
@@ -410,7 +409,7 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
     if (t < 32) {
         const int lane = t;
         // (B or E)[L][n] + n*dt, below 2^31
-        const int32_t toB = FWD ? U[skew(L)] + dt : 0;
+        const int32_t toB = FWD ? dt - U[skew(L)] : 0;  // A[L][n] + dt - Q[L] = B[L][n]
         int32_t bv = 0x7fffffff;
         int bn = 0x7fffffff;
         for (int n = 1 + lane; n <= L; n += 32) {
@@ -435,13 +434,13 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
         while (n > 1) {
             const int32_t um = U[skew(m)];
             const int32_t u = FWD ? um : um - (n - 1) * dt;
-            const int32_t target = table[tri_index(L, m, n)] + (FWD ? um + dt : 0);
+            const int32_t target = table[tri_index(L, m, n)] + (FWD ? dt : 0);  // B + Q[m] = A + dt
             const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
             int found = -1;
             for (int k0 = n - 1; k0 < m; k0 += 32) {
                 const int k = k0 + lane;
                 bool match = false;
-                if (k < m) match = cand_s32<FWD>(table[pbase + k], u, V[skew(k)]) == target;
+                if (k < m) match = cand_s32(table[pbase + k], u, V[skew(k)]) == target;
                 const unsigned bal = __ballot_sync(0xffffffffu, match);
                 if (bal) {
                     found = k0 + __ffs(bal) - 1;

@@ -7,11 +7,12 @@
 // start of the cell's last transfer, so that a transition is one 32-bit
 // add-then-max and the minimum runs on 3-input mins (1.5 integer-ALU
 // instructions per transition):
-//   forward : B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
+//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k] - dt,
 //   backward: E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),
-// with G[k] = FC[L] - FC[k], NQ[m] = -(dt + P[m]), NGT[k] = -(transfer prefix),
-// B[m][1] = FC[L], E[m][1] = BC[m]; the makespan is min_n (B or E)[L][n] + n*dt
-// plus the transfer sum. Every candidate differs from Eq. 8/9's by a constant of
+// with G[k] = FC[L] - FC[k], Q[m] = dt + P[m], NGT[k] = -(transfer prefix),
+// A[m][1] = FC[L] + P[m], E[m][1] = BC[m]; both are min_k max(u[m] + V[k], C[k])
+// with the previous column C in the max operand. The makespan is
+// min_n (B or E)[L][n] + n*dt plus the transfer sum. Every candidate differs from Eq. 8/9's by a constant of
 // its row, so every argmin is the same.
 //
 // Design (GB300):
@@ -108,18 +109,18 @@ __global__ void __launch_bounds__(32)
             for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
             continue;
         }
-        // per-layer arrays (U, V) = (NQ, G) forward, (BC, NGT) backward, written
+        // per-layer arrays (U, V) = (Q, G) forward, (BC, NGT) backward, written
         // with wrapping 32-bit arithmetic: used only when the range check passes
         uint64_t pc = 0, pxc = 0;
         const uint32_t dtu = uint32_t(dti), tcu = uint32_t(tc);
-        lw[0] = FWD ? 0u - dtu : 0u;
+        lw[0] = FWD ? dtu : 0u;
         pv[0].y = FWD ? int32_t(tcu) : 0;
         for (int r = 1; r <= L; ++r) {
             const int col = FWD ? r - 1 : L - r;
             const uint64_t cv = uint64_t(__ldg(crow + col)), xv = uint64_t(__ldg(xrow + col));
             pc += cv;
             pxc += xv < tc ? xv : tc;
-            lw[32 * r] = FWD ? 0u - dtu - uint32_t(pxc) : uint32_t(pc);
+            lw[32 * r] = FWD ? dtu + uint32_t(pxc) : uint32_t(pc);
             pv[32 * r].y = int32_t(FWD ? tcu - uint32_t(pc) : 0u - uint32_t(pxc));
         }
         if (pc + pxc + uint64_t(L) * uint64_t(dti) > kShiftedLimit) {
@@ -130,7 +131,7 @@ __global__ void __launch_bounds__(32)
 
         // ---- fill
         const int32_t dt32 = int32_t(dti), fcL = int32_t(tc);
-        for (int m = 1; m <= L; ++m) pv[32 * m].x = FWD ? fcL - U[32 * m] - dt32 : U[32 * m];
+        for (int m = 1; m <= L; ++m) pv[32 * m].x = FWD ? fcL + U[32 * m] - dt32 : U[32 * m];
         int32_t bestV = (FWD ? fcL : U[32 * L]) + dt32;
         int s = 1;
         for (int n = 2; n <= L; ++n) {
@@ -147,9 +148,7 @@ __global__ void __launch_bounds__(32)
                 }
                 // k below the block, four then two at a time: every row of the
                 // block takes them; one 64-bit load brings a (column, V) pair
-                auto cand = [&](int2 p, int j) {
-                    return FWD ? __viaddmax_s32(p.x, Ur[j], p.y) : __viaddmax_s32(Ur[j], p.y, p.x);
-                };
+                auto cand = [&](int2 p, int j) { return __viaddmax_s32(Ur[j], p.y, p.x); };
                 int k = n - 1;
                 for (; k + 3 < bot; k += 4) {
                     const int2 p0 = pv[32 * k], p1 = pv[32 * (k + 1)];
@@ -184,11 +183,11 @@ __global__ void __launch_bounds__(32)
                         for (; t + 1 < j; t += 2) best[j] = __vimin3_s32(best[j], cand(q[t], j), cand(q[t + 1], j));
                         if (t < j) best[j] = min(best[j], cand(q[t], j));
                     }
-                    if (top == L) last = best[kB - 1];
+                    if (top == L) last = FWD ? best[kB - 1] - Ur[kB - 1] : best[kB - 1];
                     const int64_t cb = int64_t(mid_cell(L, bot, n)) * nslots;
 #pragma unroll
                     for (int j = 0; j < kB; ++j) {
-                        const int32_t val = FWD ? best[j] - Ur[j] - dt32 : best[j];
+                        const int32_t val = FWD ? best[j] - dt32 : best[j];
                         pv[32 * (bot + j)].x = val;
                         if (n <= keep) myslot[cb + int64_t(j) * nslots] = uint32_t(val);
                     }
@@ -207,8 +206,8 @@ __global__ void __launch_bounds__(32)
                 for (int j = 0; j < kB; ++j) {
                     const int m = bot + j;
                     if (m <= top) {
-                        if (m == L) last = best[j];
-                        const int32_t val = FWD ? best[j] - U[32 * m] - dt32 : best[j];
+                        if (m == L) last = FWD ? best[j] - Ur[j] : best[j];
+                        const int32_t val = FWD ? best[j] - dt32 : best[j];
                         pv[32 * m].x = val;
                         if (n <= keep) myslot[int64_t(mid_cell(L, m, n)) * nslots] = uint32_t(val);
                     }
@@ -228,10 +227,10 @@ __global__ void __launch_bounds__(32)
         // ---- traceback: lowest k whose candidate equals the cell
         uint32_t word0 = 0u, word1 = 0u;  // L <= 64: W <= 2
         int err = 0, m = L, n = s;
-        int32_t target = bestV - s * dt32;  // B[L][s] or E[L][s]
+        int32_t target = bestV - s * dt32 + (FWD ? U[32 * L] : 0);  // B[L][s] + Q[L] or E[L][s]
         while (n > 1) {
             const int32_t um = U[32 * m];
-            const int32_t Rn = um - (n - 1) * dt32;  // backward only
+            const int32_t uu = FWD ? um : um - (n - 1) * dt32;
             // candidates in groups of 4 (loads issued together, lowest match wins)
             int k = -1;
             int32_t fk = 0;
@@ -242,14 +241,13 @@ __global__ void __launch_bounds__(32)
                     const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
                     v[u] = pv[32 * kk].y;
                     if (n - 1 == 1)  // column 1 is not stored
-                        f[u] = FWD ? fcL - U[32 * kk] - dt32 : U[32 * kk];
+                        f[u] = FWD ? fcL + U[32 * kk] - dt32 : U[32 * kk];
                     else
                         f[u] = int32_t(myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots]);
                 }
 #pragma unroll
                 for (int u = 3; u >= 0; --u) {
-                    const int32_t cand = FWD ? __viaddmax_s32(f[u], um, v[u]) : __viaddmax_s32(Rn, v[u], f[u]);
-                    if (k0 + u < m && cand == target) {
+                    if (k0 + u < m && __viaddmax_s32(uu, v[u], f[u]) == target) {
                         k = k0 + u;
                         fk = f[u];
                     }
@@ -263,7 +261,7 @@ __global__ void __launch_bounds__(32)
                 word0 |= 1u << (k - 1);
             else
                 word1 |= 1u << (k - 33);
-            target = FWD ? fk + U[32 * k] + dt32 : fk;  // B[k][n-1] = A + P[k]
+            target = FWD ? fk + dt32 : fk;  // the cell (k, n-1): B + Q[k] = A + dt, or E
             m = k;
             n -= 1;
         }

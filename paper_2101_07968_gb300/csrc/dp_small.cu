@@ -215,18 +215,22 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
 // costs 1.5 ALU-pipe instructions instead of 2.
 //
 // forward (P = transfer prefix, FC = compute prefix, G[k] = FC[L] - FC[k],
-// NQ[m] = -(dt + P[m])): with B = X - n*dt - P[m] + G[m] (X as above),
-//   B[m][n] = min_k max(A[k] + NQ[m], G[k]),  A[k] = B[k][n-1] - NQ[k] - dt,
-//   B[m][1] = FC[L],  X[L][n] = B[L][n] + n*dt + P[L];
+// Q[m] = dt + P[m]): with B = X - n*dt - P[m] + G[m] (X as above) and
+// A[k] = B[k][n-1] + P[k] - dt,
+//   B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[m][1] = FC[L] + P[m],
+//   X[L][n] = B[L][n] + n*dt + P[L];
+// the next column's A[m] is that minimum less dt;
 // backward (BC = compute prefix, NGT[k] = -(transfer prefix)): with
 // E = X - n*dt - S[m],
 //   E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),  E[m][1] = BC[m],
 //   X[L][n] = E[L][n] + n*dt + S[L].
-// Each candidate differs from Eq. 8/9's by a constant of its row, so every
-// argmin is the same. All values and sums lie in [-2^31, 2^31) when the capped
-// bound L*dt + sum(comp) + sum(capped xfer) is below 2^31; other instances take
-// the 64-bit pass. The table stores A (forward) or E (backward) for columns
-// 2..kKeepCols; the lane's two arrays hold NQ and G (forward) or BC and NGT.
+// Both are min_k max(u[m] + V[k], C[k]) with a row constant u and the previous
+// column C in the max operand. Each candidate differs from Eq. 8/9's by a
+// constant of its row, so every argmin is the same. All values and sums lie in
+// [-2^31, 2^31) when the capped bound L*dt + sum(comp) + sum(capped xfer) is
+// below 2^31; other instances take the 64-bit pass. The table stores A (forward)
+// or E (backward) for columns 2..kKeepCols; the lane's two arrays hold U = Q and
+// V = G (forward) or U = BC and V = NGT.
 
 // Minimum of c[0..cnt-1] (cnt a compile-time constant after unrolling): two
 // chains of 3-input mins, so that each row has two independent dependency chains
@@ -254,10 +258,10 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
                                        int &best_s)
 {
     using K = Small<L, uint32_t, kKeepCols>;
-    // forward: U = NQ, V = G, col = A; backward: U = BC, V = NGT, col = E
+    // forward: U = Q, V = G, col = A; backward: U = BC, V = NGT, col = E
     int32_t col[L + 1];
 #pragma unroll
-    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL - U[m] - dt : U[m];
+    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL + U[m] - dt : U[m];
     bestV = (FWD ? fcL : U[L]) + dt;
     best_s = 1;
 #pragma unroll
@@ -266,18 +270,13 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
 #pragma unroll
         for (int m = L; m >= n; --m) {  // descending: column n overwrites column n-1 in place
             const int cnt = m - n + 1;  // k = n-1 .. m-1
+            const int32_t u = FWD ? U[m] : U[m] - (n - 1) * dt;
             int32_t c[L];
-            if (FWD) {
 #pragma unroll
-                for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(col[n - 1 + j], U[m], V[n - 1 + j]);
-            } else {
-                const int32_t Rn = U[m] - (n - 1) * dt;
-#pragma unroll
-                for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(Rn, V[n - 1 + j], col[n - 1 + j]);
-            }
+            for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(u, V[n - 1 + j], col[n - 1 + j]);
             const int32_t b = min_fold3<L>(c, cnt);
-            if (m == L) last = b;
-            col[m] = FWD ? b - U[m] - dt : b;
+            if (m == L) last = FWD ? b - U[L] : b;
+            col[m] = FWD ? b - dt : b;
             if (n <= K::kLast) lw[32 * cell2(L, m, n)] = col[m];
         }
         const int32_t v = last + n * dt;
@@ -304,7 +303,7 @@ __device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint6
     int32_t U[L + 1], V[L + 1];
 #pragma unroll
     for (int m = 0; m <= L; ++m) {
-        U[m] = FWD ? -(dt + int32_t(Px[m])) : int32_t(Pc[m]);
+        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]);
         V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
         lw[32 * (K::kOffR + m)] = U[m];
         lw[32 * (K::kOffS + m)] = V[m];
@@ -315,44 +314,46 @@ __device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint6
     if (s - 1 > K::kLast && s - 1 >= 2) return false;
 
     // from (L, s) step to the lowest k whose candidate equals the cell, set
-    // p_k / g_k, continue at (k, n-1)
+    // p_k / g_k, continue at (k, n-1). A step compares every candidate at once
+    // (U and V still in registers, compile-time k): bit k of `hit` is set when
+    // candidate k equals the cell, and the lowest k inside [n-1, m-1] is the one
+    // Algorithm 3/4 keeps.
     uint32_t word = 0;
     int err = 0;
     int m = L, n = s;
-    int32_t target = bestV - s * dt;  // B[L][s] or E[L][s]
+    int32_t target = bestV - s * dt + (FWD ? U[L] : 0);  // B[L][s] + Q[L] or E[L][s]
     while (n > 1) {
+        const int nm1 = n - 1;
         const int32_t um = lds(lw, K::kOffR + m);
-        const int32_t Rn = um - (n - 1) * dt;  // backward only
-        int k = -1;
-        int32_t fk = 0;
-        for (int k0 = n - 1; k0 < m && k < 0; k0 += kTbGroup) {
-            int32_t f[kTbGroup], v[kTbGroup];
+        const int32_t u = FWD ? um : um - nm1 * dt;
+        uint32_t hit = 0u;
+        if (nm1 == 1) {  // column 1 is not stored: A = FC[L] + Q - dt, E = BC
 #pragma unroll
-            for (int u = 0; u < kTbGroup; ++u) {
-                const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
-                v[u] = lds(lw, K::kOffS + kk);
-                if (n - 1 == 1)  // column 1 is not stored
-                    f[u] = FWD ? fcL - lds(lw, K::kOffR + kk) - dt : lds(lw, K::kOffR + kk);
-                else
-                    f[u] = lds(lw, cell2(L, kk, n - 1));
+            for (int k = 1; k < L; ++k) {
+                const int32_t f = FWD ? fcL + U[k] - dt : U[k];
+                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
             }
+        } else {
+            const int base = cell2(L, 0, nm1);  // cell (k, n-1) is base + k
 #pragma unroll
-            for (int u = kTbGroup - 1; u >= 0; --u) {
-                const int32_t cand = FWD ? __viaddmax_s32(f[u], um, v[u]) : __viaddmax_s32(Rn, v[u], f[u]);
-                if (k0 + u < m && cand == target) {
-                    k = k0 + u;
-                    fk = f[u];
-                }
+            for (int k = 1; k < L; ++k) {
+                const int32_t f = k >= nm1 ? lds(lw, base + k) : 0;
+                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
             }
         }
-        if (k < 0) {  // cannot happen: the fill and this check use the same arithmetic
+        hit &= ((2u << (m - 1)) - 1u) & ~((1u << nm1) - 1u);  // k in [n-1, m-1]
+        if (hit == 0u) {  // cannot happen: the fill and this check use the same arithmetic
             err = 1;
             break;
         }
+        const int k = __ffs(int(hit)) - 1;
         word |= 1u << ((k - 1) & 31);
-        target = FWD ? fk + lds(lw, K::kOffR + k) + dt : fk;  // B[k][n-1] = A + P[k]
+        if (nm1 >= 2) {  // the cell (k, n-1): B + Q[k] = A + dt, or E
+            const int32_t fk = lds(lw, cell2(L, k, nm1));
+            target = FWD ? fk + dt : fk;
+        }
         m = k;
-        n -= 1;
+        n = nm1;
     }
     makespan[i] = int64_t(uint64_t(uint32_t(bestV)) + xraw);
     if (nseg) nseg[i] = s;
