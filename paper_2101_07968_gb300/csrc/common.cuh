@@ -78,6 +78,15 @@ __host__ __device__ inline bool exceeds_range(int L, int64_t dt, uint64_t sc, ui
     return tl >= lim || sc + sx + tl >= lim;
 }
 
+// Programmatic dependent launch (sm_90 and later). A kernel launched with the
+// programmatic stream serialization attribute may begin before the kernel ahead
+// of it in the stream has finished: pdl_wait() then holds its threads (a
+// hardware wait, not a spin) until that kernel has completed and its memory
+// writes are visible; pdl_trigger() in the earlier kernel lets the later one
+// start launching before the earlier one's CTAs exit.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 template <typename T>
 __device__ __forceinline__ T dmax(T a, T b) { return a > b ? a : b; }
 template <typename T>

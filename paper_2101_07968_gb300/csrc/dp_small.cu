@@ -447,6 +447,7 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
 
     const int64_t tiles = (batch + 31) / 32;
     int64_t tile = blockIdx.x;
+    pdl_trigger();  // the list pass may be scheduled as soon as CTAs of this one exit
     if (tile >= tiles) return;
     auto rows_of = [&](int64_t t) { return int(batch - t * 32 < 32 ? batch - t * 32 : 32); };
     for (; tile < tiles; tile += gridDim.x) {
@@ -497,6 +498,7 @@ __global__ void __launch_bounds__(32)
     extern __shared__ __align__(16) unsigned char smem[];
     const int lane = threadIdx.x;
     uint64_t *lw = reinterpret_cast<uint64_t *>(smem) + lane;
+    pdl_wait();  // the dense pass has finished its list
     const int64_t count = int64_t(*wide_count);
     for (int64_t j = int64_t(blockIdx.x) * 32 + lane; j - lane < count; j += int64_t(gridDim.x) * 32) {
         if (j >= count) continue;
@@ -560,13 +562,25 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
         batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    // the list length is known on the device only: size the grid for the worst
-    // case and let surplus warps exit at once
+    // the list length is known on the device only: persistent warps (4 per SM)
+    // walk it, and the surplus exits at once
     int64_t lgrid = (batch + 31) / 32;
-    if (lgrid > int64_t(sm_count()) * 8) lgrid = int64_t(sm_count()) * 8;
-    small_list_kernel<L, FWD><<<unsigned(lgrid), 32, K64::kTableBytes, stream>>>(
-        comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
-    return cudaGetLastError();
+    if (lgrid > int64_t(sm_count()) * 4) lgrid = int64_t(sm_count()) * 4;
+    // launched early (programmatic dependent launch): its CTAs wait in hardware
+    // until the dense pass completes, so the launch overlaps that pass's tail
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(unsigned(lgrid));
+    lc.blockDim = dim3(32);
+    lc.dynamicSmemBytes = K64::kTableBytes;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, small_list_kernel<L, FWD>, comp, xfer, dt, makespan, bits,
+                              nseg, status, static_cast<const uint32_t *>(wide_count),
+                              static_cast<const uint32_t *>(wide_list));
 }
 
 }  // namespace
