@@ -201,6 +201,85 @@ def run_reference(args):
     return 0
 
 
+# ------------------------------------------------------- scaling in L
+def run_lsweep(args):
+    """Scheduling time against depth L (the analogue of the paper's Fig. 12): for
+    each L, the GPU's forward + backward DP over a batch, per instance and
+    direction, beside the oracle on one host core over a sample of the same
+    instances, which are also checked bit for bit; then the log-log slope."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2101_07968_gb300 import build as libbuild
+    from paper_2101_07968_gb300 import dynacomm as dc
+
+    libbuild.build()
+    dc.lib()
+    oracle.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    rows = []
+    with ClockSampler(dev.index) as clk:
+        for L in wl.LSWEEP_LS:
+            batch = int(min(1 << 20, max(304, (1 << 36) // transitions(L))))
+            cfg = wl.lsweep_config(L, batch)
+            prof = dc.profile_gen(cfg, device=dev)
+            sch = dc.Scheduler(batch, L, device=dev)
+            pairs = ((0, ("fc", "pt")), (1, ("bc", "gt")))
+            for d, (c, x) in pairs:  # warm-up
+                sch.run(d, prof[c], prof[x], prof["dt"])
+            torch.cuda.synchronize()
+            reps = 3 if L <= 512 else 1
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                for d, (c, x) in pairs:
+                    sch.run(d, prof[c], prof[x], prof["dt"])
+            e1.record()
+            torch.cuda.synchronize()
+            gpu_s = e0.elapsed_time(e1) * 1e-3 / reps
+            got = {d: {k: v.cpu().numpy() for k, v in sch.run(d, prof[c], prof[x], prof["dt"]).items()}
+                   for d, (c, x) in pairs}
+            # the oracle (literal Algorithms 3 and 4) on one core; about L^3 / 3
+            # loop iterations per instance and direction
+            n_or = int(max(1, min(batch, 2e8 // (L ** 3 // 3 + 1))))
+            po = oracle.profile_gen(wl.with_batch(cfg, n_or))
+            t0 = time.perf_counter()
+            exp = {d: oracle.schedule_batch(d, po[c], po[x], po["dt"], nthreads=1) for d, (c, x) in pairs}
+            cpu_s = time.perf_counter() - t0
+            W = dc.words(L)
+            for d in (0, 1):
+                g = got[d]
+                bits = g["bits"].view(np.uint32)[:n_or, :W] if W else np.zeros((n_or, 0), np.uint32)
+                same = (np.array_equal(g["makespan"][:n_or], exp[d]["makespan"])
+                        and np.array_equal(g["nseg"][:n_or], exp[d]["nseg"])
+                        and np.array_equal(g["status"][:n_or], exp[d]["status"])
+                        and np.array_equal(bits, exp[d]["bits"].reshape(n_or, W)))
+                if not same:
+                    raise RuntimeError(f"GPU and oracle disagree at L={L} dir={d}")
+            rows.append({"L": L, "batch": batch,
+                         "gpu_us_per_instance_direction": gpu_s / (2 * batch) * 1e6,
+                         "gpu_transitions_per_s": 2 * transitions(L) * batch / gpu_s,
+                         "oracle_1core_us_per_instance_direction": cpu_s / (2 * n_or) * 1e6,
+                         "oracle_sample": n_or, "parity_checked": n_or})
+
+    def slope(key, lo):
+        pts = [(np.log(r["L"]), np.log(r[key])) for r in rows if r["L"] >= lo]
+        return float(np.polyfit([p[0] for p in pts], [p[1] for p in pts], 1)[0])
+
+    line = {"mode": "lsweep", "metric": "scheduling time per instance and direction against L",
+            "unit": "us", "higher_is_better": False, "data": "synthetic",
+            "config": {"workload": "deep-chain draws at depth L (seed 5)",
+                       "batch": "min(2^20, max(304, 2^36 / C(L)))"},
+            "rows": rows,
+            "slope_gpu_L_ge_256": slope("gpu_us_per_instance_direction", 256),
+            "slope_oracle_L_ge_128": slope("oracle_1core_us_per_instance_direction", 128),
+            "parity": "GPU outputs bit-exact with the oracle on every sampled instance, both directions",
+            "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # --------------------------------------------------------------- GPU arm
 def run_ours(args):
     import numpy as np
@@ -428,7 +507,11 @@ def main(argv=None):
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--e2e-chunks", type=int, default=8)
+    p.add_argument("--lsweep", action="store_true",
+                   help="scheduling time against depth L (GPU and one oracle core), one JSON line")
     args = p.parse_args(argv)
+    if args.lsweep:
+        return run_lsweep(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

@@ -36,7 +36,7 @@ inline int64_t table_slots(int L)
 {
     const int64_t per = tri_cells(L) * 8;
     int64_t s = (int64_t(4) << 30) / per;
-    if (s > 1024) s = 1024;
+    if (s > 152 * 32) s = 152 * 32;  // up to 32 one-warp CTAs per SM
     if (s < 152) s = 152;
     return s;
 }

@@ -931,12 +931,9 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
     }
 }
 
-int group_threads(int L)
-{
-    if (L <= 64) return 64;
-    if (L <= 256) return 128;
-    return 256;
-}
+// Threads per instance: up to L = 256 a column has few (8 x 64) tiles, so one
+// warp per instance and more instances per SM; deeper chains fill 8 warps.
+int group_threads(int L) { return L <= 256 ? 32 : 256; }
 
 }  // namespace
 

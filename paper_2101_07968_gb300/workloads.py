@@ -119,6 +119,18 @@ def config(name: str) -> dict:
 
 CONFIG_NAMES = ("tiny", "alexnet", "vgg16", "resnet50", "deepchain")
 
+# Depths of the scheduling-time-versus-L sweep (the paper's Fig. 12 times its
+# schedulers on randomly generated profiles of growing depth).
+LSWEEP_LS = (8, 16, 32, 64, 128, 256, 512, 1024, 2048)
+
+
+def lsweep_config(L: int, batch: int, seed: int = 5) -> dict:
+    """The deep-chain draws (per-instance log-uniform params and FLOPs per layer,
+    per-instance rate, bandwidth and latency) at depth L."""
+    c = config("deepchain")
+    c.update(name=f"lsweep{L}", L=int(L), batch=int(batch), seed=int(seed))
+    return c
+
 
 def with_batch(cfg: dict, batch: int, inst0: int = 0) -> dict:
     c = dict(cfg)

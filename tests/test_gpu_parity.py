@@ -256,6 +256,22 @@ def test_config_deepchain_sampled_parity(dc):
     _config_parity(dc, "deepchain", sample=sample)
 
 
+@pytest.mark.parametrize("L,sample", [(256, 64), (512, 16), (2048, 2)])
+def test_lsweep_sampled_parity(dc, L, sample):
+    """The depth sweep's inputs (deep-chain draws at depth L) over several CTAs'
+    worth of instances: a sample bit-exact with the oracle, every decision replayed."""
+    B = 304
+    cfg = wl.lsweep_config(L, B)
+    prof = oracle.profile_gen(cfg)
+    for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+        got = _gpu_schedule(dc, d, prof[c], prof[x], prof["dt"])
+        exp = oracle.schedule_batch(d, prof[c][:sample], prof[x][:sample], prof["dt"][:sample],
+                                    nthreads=NTHREADS)
+        _assert_same({k: v[:sample] for k, v in got.items()}, exp, f"lsweep L={L} dir={d}")
+        rep = oracle.replay_batch(d, prof[c], prof[x], prof["dt"], got["bits"], nthreads=NTHREADS)
+        assert np.array_equal(rep, got["makespan"])
+
+
 def test_roof_probe_runs(dc):
     import torch
     sink = torch.empty(152 * 256, dtype=torch.int32, device="cuda")
