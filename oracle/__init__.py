@@ -2,8 +2,9 @@
 
 A plain C transcription of the paper's scheduling path (Algorithm 3 / Eq. 8,
 Algorithm 4 / Eq. 9, the cost function f_m of Sec. III-B written from Eq. 1-7,
-brute force over the 0-1 program, and the seeded profile generator standing in
-for the profiler of Sec. IV-A), wrapped with ctypes and numpy.
+brute force over the 0-1 program, the seeded profile generator standing in
+for the profiler of Sec. IV-A, and the paper's competing greedy schedulers,
+Algorithms 1 and 2), wrapped with ctypes and numpy.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg
 may import this package. It shares no code with the CUDA library in
@@ -19,6 +20,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "dynacomm_oracle.c")
+_SRC_GREEDY = os.path.join(_HERE, "greedy_oracle.c")
 _HDR = os.path.join(_HERE, "dynacomm_oracle.h")
 _LIB = os.path.join(_HERE, "liboracle.so")
 
@@ -29,11 +31,11 @@ DIST_UNIFORM, DIST_LOGUNIFORM = 0, 1
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (plain C99, -O2, pthreads)."""
     stale = force or not os.path.exists(_LIB) or any(
-        os.path.getmtime(p) > os.path.getmtime(_LIB) for p in (_SRC, _HDR))
+        os.path.getmtime(p) > os.path.getmtime(_LIB) for p in (_SRC, _SRC_GREEDY, _HDR))
     if stale:
         tmp = _LIB + f".tmp{os.getpid()}"
         subprocess.check_call(["gcc", "-std=gnu99", "-O2", "-fPIC", "-shared", "-Wall",
-                               "-o", tmp, _SRC, "-lm", "-lpthread"])
+                               "-o", tmp, _SRC, _SRC_GREEDY, "-lm", "-lpthread"])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -89,6 +91,12 @@ def lib():
         _lib.orc_instance_draws.argtypes = [ctypes.POINTER(_Cfg), i64, vp, vp, vp]
         _lib.orc_layer_draw.restype = i64
         _lib.orc_layer_draw.argtypes = [ctypes.POINTER(_Cfg), i64, i32, i32]
+        _lib.orc_greedy_forward.restype = None
+        _lib.orc_greedy_forward.argtypes = [i32, vp, vp, i64, vp]
+        _lib.orc_greedy_backward.restype = None
+        _lib.orc_greedy_backward.argtypes = [i32, vp, vp, i64, vp]
+        _lib.orc_greedy_batch.restype = None
+        _lib.orc_greedy_batch.argtypes = [i32, i64, i32, vp, vp, vp, vp, vp, i32]
         _lib.orc_profile_gen.restype = i32
         _lib.orc_profile_gen.argtypes = [ctypes.POINTER(_Cfg), vp, vp, vp, vp, vp]
     return _lib
@@ -173,6 +181,35 @@ def replay_batch(direction: int, comp, xfer, dt, bits, nthreads: int = 1) -> np.
     out = np.zeros(B, np.int64)
     lib().orc_replay_batch(direction, B, L, _p(comp), _p(xfer), _p(dt), _p(bits), _p(out),
                            int(nthreads))
+    return out
+
+
+def greedy_forward(pt, fc, dt: int) -> np.ndarray:
+    """Algorithm 1 (iBatch forward greedy): decision p[0..L] (uint8)."""
+    pt, fc = _i64(pt), _i64(fc)
+    L = len(pt)
+    p = np.zeros(L + 1, np.uint8)
+    lib().orc_greedy_forward(L, _p(pt), _p(fc), int(dt), _p(p))
+    return p
+
+
+def greedy_backward(bc, gt, dt: int) -> np.ndarray:
+    """Algorithm 2 (iPart backward greedy): decision g[0..L] (uint8)."""
+    bc, gt = _i64(bc), _i64(gt)
+    L = len(bc)
+    g = np.zeros(L + 1, np.uint8)
+    lib().orc_greedy_backward(L, _p(bc), _p(gt), int(dt), _p(g))
+    return g
+
+
+def greedy_batch(direction: int, comp, xfer, dt, nthreads: int = 1) -> dict:
+    """Algorithm 1 (direction 0) or 2 (direction 1) over a batch: dict(bits [B,W]
+    uint32, makespan [B] int64 = f_m of the decision, -status on a bad instance)."""
+    comp, xfer, dt = _i64(comp), _i64(xfer), _i64(dt)
+    B, L = comp.shape
+    out = dict(bits=np.zeros((B, words(L)), np.uint32), makespan=np.zeros(B, np.int64))
+    lib().orc_greedy_batch(direction, B, L, _p(comp), _p(xfer), _p(dt), _p(out["bits"]),
+                           _p(out["makespan"]), int(nthreads))
     return out
 
 

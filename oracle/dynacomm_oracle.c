@@ -374,6 +374,33 @@ static void run_split(batch_job base, int64_t batch, int32_t nthreads, void *(*f
     for (int32_t t = 0; t < nthreads; t++) pthread_join(th[t], NULL);
 }
 
+static void *greedy_range(void *arg)
+{
+    batch_job *j = (batch_job *)arg;
+    uint8_t *d = (uint8_t *)malloc((size_t)j->L + 1);
+    for (int64_t i = j->lo; i < j->hi; i++) {
+        const int64_t *c = j->comp + i * j->L, *x = j->xfer + i * j->L;
+        uint32_t *w = j->bits + i * j->W;
+        for (int32_t q = 0; q < j->W; q++) w[q] = 0;
+        int32_t st = instance_status(j->L, c, x, j->dt[i]);
+        if (st != ORC_OK) {
+            j->makespan[i] = -(int64_t)st;
+            continue;
+        }
+        if (j->dir == 0)
+            orc_greedy_forward(j->L, x, c, j->dt[i], d);
+        else
+            orc_greedy_backward(j->L, c, x, j->dt[i], d);
+        d[0] = 0;
+        d[j->L] = 0;
+        for (int32_t l = 1; l <= j->L - 1; l++)
+            if (d[l]) w[(l - 1) / 32] |= 1u << ((l - 1) % 32);
+        j->makespan[i] = replay_dir(j->dir, j->L, c, x, j->dt[i], d);
+    }
+    free(d);
+    return NULL;
+}
+
 void orc_schedule_batch(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,
                         const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                         uint32_t *bits, int32_t *nseg, int32_t *status, int32_t nthreads)
@@ -536,4 +563,21 @@ int32_t orc_profile_gen(const orc_profile_cfg *cfg, int64_t *fc, int64_t *pt, in
         }
     }
     return 0;
+}
+
+void orc_greedy_batch(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,
+                      const int64_t *xfer, const int64_t *dt, uint32_t *bits, int64_t *makespan,
+                      int32_t nthreads)
+{
+    batch_job b;
+    memset(&b, 0, sizeof b);
+    b.dir = dir;
+    b.L = L;
+    b.W = (L - 1 + 31) / 32;
+    b.comp = comp;
+    b.xfer = xfer;
+    b.dt = dt;
+    b.makespan = makespan;
+    b.bits = bits;
+    run_split(b, batch, nthreads, greedy_range);
 }

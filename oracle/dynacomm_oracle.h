@@ -11,7 +11,9 @@
  *   - brute force over all 2^(L-1) decisions (Sec. III-B, the O(L 2^L) search),
  *   - an O(L^2) one-dimensional backward DP used as an independent value check,
  *   - the seeded synthetic profile generator that stands in for the real-time
- *     profiler of Sec. IV-A.
+ *     profiler of Sec. IV-A,
+ *   - the paper's competing greedy schedulers, Algorithm 1 (forward) and
+ *     Algorithm 2 (backward), in greedy_oracle.c.
  *
  * Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may load
  * this library. It shares no code, header or table with the CUDA library.
@@ -80,6 +82,19 @@ void orc_schedule_batch(int32_t dir, int64_t batch, int32_t L, const int64_t *co
 void orc_replay_batch(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,
                       const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                       int64_t *makespan, int32_t nthreads);
+
+/* ---- the paper's competing greedy schedulers (greedy_oracle.c) -------- */
+
+/* Algorithm 1 (iBatch, forward): writes p[0..L]. */
+void orc_greedy_forward(int32_t L, const int64_t *pt, const int64_t *fc, int64_t dt, uint8_t *p);
+/* Algorithm 2 (iPart, backward): writes g[0..L], g[r] = break after the last r layers. */
+void orc_greedy_backward(int32_t L, const int64_t *bc, const int64_t *gt, int64_t dt, uint8_t *g);
+/* Either over a batch: packed decisions bits [batch][W] and their f_m makespan
+ * (-status for a failed instance, with zero bits). dir 0: comp = fc, xfer = pt;
+ * dir 1: comp = bc, xfer = gt. */
+void orc_greedy_batch(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,
+                      const int64_t *xfer, const int64_t *dt, uint32_t *bits, int64_t *makespan,
+                      int32_t nthreads);
 
 /* ---- synthetic profile generator (stand-in for Sec. IV-A's profiler) ---- */
 
