@@ -148,6 +148,31 @@ dc_status dc_schedule_backward_batch(int64_t batch, int32_t L, const int64_t *bc
                                      cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * dc_greedy_forward_batch, dc_greedy_backward_batch -- the paper's competing
+ * schedulers (Sec. II-C), for comparison with the DP: greedy parameter
+ * scheduling of iBatch (Algorithm 1, forward; inputs as
+ * dc_schedule_forward_batch) and greedy gradient scheduling of iPart
+ * (Algorithm 2, backward; inputs as dc_schedule_backward_batch). Readings of the
+ * listings' open points: ties keep the first candidate of the listing's
+ * enumeration; an empty Options set takes the position with the largest slack;
+ * Algorithm 1's first pair is the qualifying pair with the largest first-segment
+ * compute, then the smallest first transfer, then the smallest slack (with no
+ * qualifying pair, the largest slack); Algorithm 2 keeps the candidate with the
+ * least f_m. Outputs per instance: bits [batch][W] (the decision, same layout
+ * as dc_schedule_*) and makespan [batch] (f_m of that decision, as
+ * dc_eval_timeline_batch gives it), or -(status) and zero bits for an instance
+ * with a negative or out-of-range input (status 3 or 4). No workspace. Errors:
+ * DC_ERR_NULL, DC_ERR_BAD_SHAPE (batch < 0 or > 2^32-1, L outside [1, 4096]),
+ * DC_ERR_CUDA. Asynchronous on `stream`.
+ * ---------------------------------------------------------------------- */
+dc_status dc_greedy_forward_batch(int64_t batch, int32_t L, const int64_t *fc, const int64_t *pt,
+                                  const int64_t *dt, int64_t *makespan, uint32_t *bits,
+                                  cudaStream_t stream);
+dc_status dc_greedy_backward_batch(int64_t batch, int32_t L, const int64_t *bc, const int64_t *gt,
+                                   const int64_t *dt, int64_t *makespan, uint32_t *bits,
+                                   cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * dc_eval_timeline_batch -- the cost measurement f_m of Sec. III-B for one
  * direction: replays ANY decision (bits [batch][W]) under the partial orders of
  * Eq. 1-7 and writes its makespan. dir 0: comp = fc, xfer = pt, the pulls run

@@ -62,6 +62,8 @@ _SIGNATURES = {
     "dc_eval_timeline_batch": (_I32, [_I64, _I32, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_schedule_batch_static": (_I32, [_I32, _I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
                                         _VP]),
+    "dc_greedy_forward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
+    "dc_greedy_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_status_string": (ctypes.c_char_p, [_I32]),
     "dc_roof_int_probe": (_I32, [_I32, _I32, _I32, _I64, _VP, _VP]),
 }
@@ -190,6 +192,16 @@ def dc_eval_timeline_batch(batch, L, direction, comp, xfer, dt, bits, makespan,
         _ptr(makespan), _stream(stream)))
 
 
+def dc_greedy_forward_batch(batch, L, fc, pt, dt, makespan, bits, stream=None) -> int:
+    return int(lib().dc_greedy_forward_batch(int(batch), int(L), _ptr(fc), _ptr(pt), _ptr(dt),
+                                             _ptr(makespan), _ptr(bits), _stream(stream)))
+
+
+def dc_greedy_backward_batch(batch, L, bc, gt, dt, makespan, bits, stream=None) -> int:
+    return int(lib().dc_greedy_backward_batch(int(batch), int(L), _ptr(bc), _ptr(gt), _ptr(dt),
+                                              _ptr(makespan), _ptr(bits), _stream(stream)))
+
+
 def dc_roof_int_probe(variant, blocks, threads, iters, sink, stream=None) -> int:
     return int(lib().dc_roof_int_probe(int(variant), int(blocks), int(threads), int(iters),
                                        _ptr(sink), _stream(stream)))
@@ -251,6 +263,21 @@ def eval_timeline(direction: int, comp, xfer, dt, bits, stream=None):
     out = torch.empty(B, dtype=torch.int64, device=comp.device)
     _check(dc_eval_timeline_batch(B, L, direction, comp, xfer, dt, bits, out, stream),
            "dc_eval_timeline_batch")
+    return out
+
+
+def greedy(direction: int, comp, xfer, dt, stream=None) -> dict:
+    """The paper's competing greedy scheduler for one direction (Algorithm 1
+    forward, Algorithm 2 backward): dict(makespan [B] int64, bits [B, max(W,1)]
+    int32 view of the uint32 decision words)."""
+    import torch
+    B, L = comp.shape
+    W = words(L)
+    out = {"makespan": torch.empty(B, dtype=torch.int64, device=comp.device),
+           "bits": torch.empty((B, max(W, 1)), dtype=torch.int32, device=comp.device)}
+    fn = dc_greedy_forward_batch if direction == 0 else dc_greedy_backward_batch
+    _check(fn(B, L, comp, xfer, dt, out["makespan"], out["bits"], stream),
+           "dc_greedy_forward_batch" if direction == 0 else "dc_greedy_backward_batch")
     return out
 
 
