@@ -280,6 +280,119 @@ def run_lsweep(args):
     return 0
 
 
+# ------------------------------------------------- competing strategies
+def run_compare(args):
+    """DynaComm's optimum against the paper's competing strategies on one
+    workload (the analogue of Figs. 5-6 on synthetic profiles): Sequential (one
+    transmission), layer by layer (LBL), the greedy schedulers (Algorithm 1
+    forward, Algorithm 2 backward), all on the GPU. Per direction: each
+    strategy's makespan over the DP optimum (distribution), the share of
+    instances where it is optimal, the running-time reduction against
+    Sequential, and each strategy's own throughput."""
+    import numpy as np
+    import torch
+
+    from paper_2101_07968_gb300 import build as libbuild
+    from paper_2101_07968_gb300 import dynacomm as dc
+
+    libbuild.build()
+    dc.lib()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    cfg = wl.config(args.workload)
+    if args.batch:
+        cfg = wl.with_batch(cfg, args.batch)
+    B, L = cfg["batch"], cfg["L"]
+    W = dc.words(L)
+    prof = dc.profile_gen(cfg, device=dev)
+    zeros = torch.zeros((B, max(W, 1)), dtype=torch.int32, device=dev)
+    ones = torch.zeros((B, max(W, 1)), dtype=torch.int32, device=dev)
+    for l in range(1, L):  # p_l / g_l = 1 for every position: layer by layer
+        bit = 1 << ((l - 1) % 32)
+        ones[:, (l - 1) // 32] |= bit - (1 << 32) if bit >= 1 << 31 else bit
+    sch = dc.Scheduler(B, L, device=dev)
+
+    def timed(fn, reps=5):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            out = fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return out, e0.elapsed_time(e1) / reps * 1e-3
+
+    result, result_mk = {}, {}
+    with ClockSampler(dev.index) as clk:
+        for d, name, (c, x) in ((0, "forward", ("fc", "pt")), (1, "backward", ("bc", "gt"))):
+            a = (prof[c], prof[x], prof["dt"])
+            dp, t_dp = timed(lambda: sch.run(d, *a)["makespan"].clone())
+            gr, t_gr = timed(lambda: dc.greedy(d, *a)["makespan"])
+            sq, t_sq = timed(lambda: dc.eval_timeline(d, *a, zeros[:, :W].contiguous() if W else None))
+            lb, t_lb = timed(lambda: dc.eval_timeline(d, *a, ones[:, :W].contiguous() if W else None))
+            opt = dp.double()
+            result_mk[name] = {"dynacomm": dp, "greedy": gr, "sequential": sq, "lbl": lb}
+            rows = {}
+            for sname, v, t in (("dynacomm", dp, t_dp), ("greedy", gr, t_gr),
+                                ("sequential", sq, t_sq), ("lbl", lb, t_lb)):
+                r = (v.double() / opt).cpu().numpy()
+                rows[sname] = {
+                    "makespan_over_optimum": {"mean": float(r.mean()), "p50": float(np.median(r)),
+                                              "p90": float(np.percentile(r, 90)),
+                                              "p99": float(np.percentile(r, 99)),
+                                              "max": float(r.max())},
+                    "optimal_share": float((v == dp).double().mean().item()),
+                    "mean_reduction_vs_sequential": float(1.0 - (v.double() / sq.double()).mean().item()),
+                    "instances_per_s": B / t}
+            result[name] = rows
+        # whole iteration (Sec. III-A: the backward pass starts after the forward)
+        it = {}
+        seq_it = result_mk["forward"]["sequential"] + result_mk["backward"]["sequential"]
+        for sname in ("dynacomm", "greedy", "sequential", "lbl"):
+            tot = result_mk["forward"][sname] + result_mk["backward"][sname]
+            it[sname] = {"mean_us": float(tot.double().mean().item()),
+                         "mean_reduction_vs_sequential": float(1.0 - (tot.double() / seq_it.double()).mean().item()),
+                         "max_reduction_vs_sequential": float(1.0 - (tot.double() / seq_it.double()).min().item())}
+        # idle windows (Sec. IV-C): the forward schedule of the next iteration can
+        # run during the last push (dt + gt of layer 1), the backward schedule
+        # during the first pull (dt + pt of layer 1); the GPU's latency for one
+        # instance, launch included, against them
+        lat = {}
+        sch1 = dc.Scheduler(1, L, device=dev)
+        for d, (c, x) in ((0, ("fc", "pt")), (1, ("bc", "gt"))):
+            a1 = (prof[c][:1], prof[x][:1], prof["dt"][:1])
+            ts = []
+            for _ in range(25):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                sch1.run(d, *a1)
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1) * 1e3)
+            lat[d] = float(np.median(ts[5:]))
+        win_f = (prof["dt"] + prof["gt"][:, 0]).double()  # hides the forward schedule
+        win_b = (prof["dt"] + prof["pt"][:, 0]).double()  # hides the backward schedule
+        window = {"single_instance_latency_us": {"forward": lat[0], "backward": lat[1]},
+                  "window_fwd_us_p01_p50": [float(torch.quantile(win_f, 0.01)), float(win_f.median())],
+                  "window_bwd_us_p01_p50": [float(torch.quantile(win_b, 0.01)), float(win_b.median())],
+                  "hidden_share_forward": float((win_f >= lat[0]).double().mean()),
+                  "hidden_share_backward": float((win_b >= lat[1]).double().mean()),
+                  "batch_amortised_us_per_instance": {
+                      "forward": 1e6 / result["forward"]["dynacomm"]["instances_per_s"],
+                      "backward": 1e6 / result["backward"]["dynacomm"]["instances_per_s"]}}
+    line = {"mode": "compare", "metric": "makespan of each strategy over the DP optimum",
+            "data": "synthetic", "config": {"workload": args.workload, "batch": B, "L": L},
+            "iteration": it, "idle_window": window,
+            "strategies": {"dynacomm": "Algorithms 3/4 (dc_schedule_*)",
+                           "greedy": "Algorithm 1 forward / Algorithm 2 backward (dc_greedy_*)",
+                           "sequential": "one transmission (dc_eval_timeline_batch, no break)",
+                           "lbl": "layer by layer (dc_eval_timeline_batch, every break)"},
+            "result": result, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # --------------------------------------------------------------- GPU arm
 def run_ours(args):
     import numpy as np
@@ -509,9 +622,13 @@ def main(argv=None):
     p.add_argument("--e2e-chunks", type=int, default=8)
     p.add_argument("--lsweep", action="store_true",
                    help="scheduling time against depth L (GPU and one oracle core), one JSON line")
+    p.add_argument("--compare", action="store_true",
+                   help="DynaComm against Sequential, LBL and the greedy schedulers, one JSON line")
     args = p.parse_args(argv)
     if args.lsweep:
         return run_lsweep(args)
+    if args.compare:
+        return run_compare(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
