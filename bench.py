@@ -393,6 +393,72 @@ def run_compare(args):
     return 0
 
 
+# ------------------------------------------------- fused generate-and-solve
+def run_fused(args):
+    """Generate-and-solve in one pass (dc_schedule_generated_batch, L <= 16)
+    against the unfused dc_profile_gen + forward DP + backward DP on the same
+    workload: the same results bit for bit (checked here), without the profiles'
+    round trip through HBM. Reported separately from the step: fusion changes
+    the algorithmic byte count."""
+    import torch
+
+    from paper_2101_07968_gb300 import build as libbuild
+    from paper_2101_07968_gb300 import dynacomm as dc
+
+    libbuild.build()
+    dc.lib()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    cfg = wl.config(args.workload)
+    if args.batch:
+        cfg = wl.with_batch(cfg, args.batch)
+    B, L = cfg["batch"], cfg["L"]
+    W = dc.words(L)
+    fused = dc.GeneratedScheduler(cfg, device=dev)
+    prof = {k: torch.empty((B, L), dtype=torch.int64, device=dev) for k in ("fc", "pt", "bc", "gt")}
+    prof["dt"] = torch.empty(B, dtype=torch.int64, device=dev)
+    sch = dc.Scheduler(B, L, device=dev)
+    keep: list = []
+    ccfg = dc.make_cfg(cfg, keep)
+
+    def unfused():
+        assert dc.dc_profile_gen(ccfg, prof["fc"], prof["pt"], prof["bc"], prof["gt"], prof["dt"]) == 0
+        return [sch.run(d, prof[c], prof[x], prof["dt"])["makespan"]
+                for d, (c, x) in ((0, ("fc", "pt")), (1, ("bc", "gt")))]
+
+    def timed(fn, reps):
+        for _ in range(max(args.warmup, 3)):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    with ClockSampler(dev.index) as clk:
+        ms_f = timed(fused.run, args.steps)
+        ms_u = timed(unfused, args.steps)
+    fo = fused.run()
+    mk = unfused()
+    torch.cuda.synchronize()
+    same = all(torch.equal(fo["makespan"][d], mk[d]) for d in (0, 1))
+    if not same:
+        raise RuntimeError("fused and unfused results differ")
+    out_b = 2 * (8 + 4 * W + 4 + 4)
+    line = {"mode": "fused", "metric": "generate + forward DP + backward DP, instances/s",
+            "unit": "instances/s", "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": args.workload, "batch": B, "L": L},
+            "fused": {"value": B / (ms_f * 1e-3), "ms": ms_f,
+                      "algorithmic_bytes_per_instance": out_b},
+            "unfused": {"value": B / (ms_u * 1e-3), "ms": ms_u,
+                        "algorithmic_bytes_per_instance": (4 * L + 1) * 8 + 2 * (2 * L * 8 + 8) + out_b},
+            "speedup": ms_u / ms_f, "bit_exact": same, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # --------------------------------------------------------------- GPU arm
 def run_ours(args):
     import numpy as np
@@ -624,7 +690,11 @@ def main(argv=None):
                    help="scheduling time against depth L (GPU and one oracle core), one JSON line")
     p.add_argument("--compare", action="store_true",
                    help="DynaComm against Sequential, LBL and the greedy schedulers, one JSON line")
+    p.add_argument("--fused", action="store_true",
+                   help="generate-and-solve in one pass against the unfused path (L <= 16)")
     args = p.parse_args(argv)
+    if args.fused:
+        return run_fused(args)
     if args.lsweep:
         return run_lsweep(args)
     if args.compare:

@@ -148,6 +148,25 @@ dc_status dc_schedule_backward_batch(int64_t batch, int32_t L, const int64_t *bc
                                      cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * dc_schedule_generated_batch -- dc_profile_gen followed by both
+ * dc_schedule_forward_batch and dc_schedule_backward_batch for 1 <= L <= 16,
+ * fused: every instance's profile is drawn inside the solving kernel (the same
+ * pure function of seed, instance, field and layer that dc_profile_gen writes
+ * out) and never stored, so the profiles make no round trip through device
+ * memory. The results are those of the unfused calls on dc_profile_gen's output,
+ * bit for bit. Outputs, forward first then backward: makespan [2][batch],
+ * bits [2][batch][W], nseg [2][batch] and status [2][batch] (both nullable).
+ * workspace: device, >= dc_schedule_generated_workspace_bytes(batch, L) bytes
+ * (the two work lists and a copy of the generator's tables). Errors: those of dc_profile_gen (config), DC_ERR_BAD_SHAPE
+ * for L > 16, DC_ERR_NULL, DC_ERR_WORKSPACE, DC_ERR_CUDA. There is no counterpart
+ * in the paper, whose profiler produces the profiles (Sec. IV-A).
+ * ---------------------------------------------------------------------- */
+size_t dc_schedule_generated_workspace_bytes(int64_t batch, int32_t L);
+dc_status dc_schedule_generated_batch(const dc_profile_cfg *cfg, int64_t *makespan, uint32_t *bits,
+                                      int32_t *nseg, int32_t *status, void *workspace,
+                                      size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * dc_greedy_forward_batch, dc_greedy_backward_batch -- the paper's competing
  * schedulers (Sec. II-C), for comparison with the DP: greedy parameter
  * scheduling of iBatch (Algorithm 1, forward; inputs as

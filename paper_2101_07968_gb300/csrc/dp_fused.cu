@@ -1,0 +1,250 @@
+// Generate-and-solve for 1 <= L <= 16 (dc_schedule_generated_batch): the short-L
+// passes of dp_small.cu with each tile's rows drawn inside the kernel by the
+// profile generator's device functions instead of being read from memory.
+#include "dp_small.cuh"
+
+namespace dc {
+namespace {
+
+// ---------------------------------------------------------------------------
+// Generate and solve in one pass (no profile round trip through HBM): each lane
+// draws its instance's rows with the profile generator's own device functions
+// into its row of the staging area, then the tile is solved as in dp_small.cu;
+// one pass per direction, each with its own list pass, which regenerates the
+// listed instances' rows.
+// workspace: [0, 256) the two list counters, [256, 256 + 8 batch) the two lists,
+// then the generator's tables
+inline size_t fused_tables_offset(int64_t batch) { return (256 + 8 * size_t(batch) + 255) / 256 * 256; }
+
+struct FusedOut {
+    int64_t *makespan[2];
+    uint32_t *bits[2];
+    int32_t *nseg[2], *status[2];
+    uint32_t *wide_count[2], *wide_list[2];
+};
+
+// The generator's lookup tables, copied once per call from the parameter block
+// into the workspace: lanes index them with their own draws, which global loads
+// serve in parallel where the parameter (constant) path serialises them.
+struct GenTables {
+    int64_t rate[kKnots + 1], bw[kKnots + 1], l0[kFixedMax], l1[kFixedMax];
+};
+
+__global__ void __launch_bounds__(256) copy_tables_kernel(const __grid_constant__ GenParams g,
+                                                          GenTables *t)
+{
+    for (int j = threadIdx.x; j <= kKnots; j += blockDim.x) {
+        t->rate[j] = g.rate_knots[j];
+        t->bw[j] = g.bw_knots[j];
+    }
+    for (int j = threadIdx.x; j < kFixedMax; j += blockDim.x) {
+        t->l0[j] = g.layer0[j];
+        t->l1[j] = g.layer1[j];
+    }
+}
+
+template <int L, bool FWD>
+__device__ __forceinline__ void fused_direction(const GenParams &g, const GenTables *t,
+                                                const InstanceDraws &d,
+                                                int64_t gi, int64_t i, bool active, int64_t *stC,
+                                                int64_t *stX, int32_t *lw, int lane,
+                                                const FusedOut &o)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    constexpr int W = (L - 1 + 31) / 32;
+    constexpr int dir = FWD ? 0 : 1;
+    __syncwarp();  // every lane is done with the area (the table of the other direction)
+    if (active) {
+#pragma unroll
+        for (int l = 0; l < L; ++l) {
+            int64_t params, flops, f, b, x;
+            layer_draws(g, t->l0, t->l1, gi, l, params, flops);
+            layer_costs(g, d, params, flops, f, b, x);
+            stC[lane * K::kStride + l] = FWD ? f : b;
+            stX[lane * K::kStride + l] = x;
+        }
+    }
+    const int64_t dti = active ? d.dt : 0;
+    uint64_t Pc[L + 1], Px[L + 1], xraw;
+    bool neg = dti < 0, big = (dti >> 52) != 0;
+    row_prefix<L, FWD>(
+        [&](int col, int64_t &cv, int64_t &xv) {
+            cv = active ? stC[lane * K::kStride + col] : 0;
+            xv = active ? stX[lane * K::kStride + col] : 0;
+        },
+        Pc, Px, xraw, neg, big);
+    __syncwarp();  // rows read: the lanes' table slices may be written
+    if (!active) return;
+    int st = DC_OK;
+    if (neg)
+        st = DC_ERR_NEGATIVE;
+    else if (big || uint64_t(L) * uint64_t(dti) + Pc[L] + xraw >= uint64_t(kRangeLimit))
+        st = DC_ERR_RANGE;
+    const uint64_t bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];  // capped
+    if (st != DC_OK) {
+        write_failure(st, i, W, o.makespan[dir], o.bits[dir], o.nseg[dir], o.status[dir]);
+    } else if (bound > kShiftedLimit ||
+               !solve_e<L, FWD>(Pc, Px, dti, xraw, lw, i, o.makespan[dir], o.bits[dir],
+                                o.nseg[dir], o.status[dir])) {
+        o.wide_list[dir][atomicAdd(o.wide_count[dir], 1u)] = uint32_t(i);
+    }
+}
+
+template <int L, bool FWD>
+__global__ void __launch_bounds__(32, DC_SMALL_MINB)
+    fused_dense_kernel(const __grid_constant__ GenParams g, const GenTables *t, const FusedOut o)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x;
+    int64_t *stC = reinterpret_cast<int64_t *>(smem);
+    int64_t *stX = stC + 32 * K::kStride;
+    int32_t *lw = reinterpret_cast<int32_t *>(smem) + lane;
+    const int64_t tiles = (g.batch + 31) / 32;
+    int64_t tile = blockIdx.x;
+    pdl_trigger();
+    if (tile >= tiles) return;
+    for (; tile < tiles; tile += gridDim.x) {
+        const int64_t i = tile * 32 + lane;
+        const bool active = i < g.batch;
+        const int64_t gi = g.inst0 + i;
+        InstanceDraws d = {};
+        if (active) d = instance_draws(g, t->rate, t->bw, gi);
+        fused_direction<L, FWD>(g, t, d, gi, i, active, stC, stX, lw, lane, o);
+    }
+}
+
+// 64-bit pass over one direction's list, rows regenerated.
+template <int L, bool FWD>
+__global__ void __launch_bounds__(32)
+    fused_list_kernel(const __grid_constant__ GenParams g, const GenTables *t, const FusedOut o)
+{
+    constexpr int dir = FWD ? 0 : 1;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x;
+    uint64_t *lw = reinterpret_cast<uint64_t *>(smem) + lane;
+    pdl_wait();  // the passes ahead of this one have finished
+    const int64_t count = int64_t(*o.wide_count[dir]);
+    for (int64_t j = int64_t(blockIdx.x) * 32 + lane; j - lane < count; j += int64_t(gridDim.x) * 32) {
+        if (j >= count) continue;
+        const int64_t i = int64_t(o.wide_list[dir][j]);
+        const int64_t gi = g.inst0 + i;
+        const InstanceDraws d = instance_draws(g, t->rate, t->bw, gi);
+        uint64_t Pc[L + 1], Px[L + 1], xraw;
+        bool neg = false, big = false;  // checked by the dense pass
+        row_prefix<L, FWD>(
+            [&](int col, int64_t &cv, int64_t &xv) {
+                int64_t params, flops, f, b, x;
+                layer_draws(g, t->l0, t->l1, gi, col, params, flops);
+                layer_costs(g, d, params, flops, f, b, x);
+                cv = FWD ? f : b;
+                xv = x;
+            },
+            Pc, Px, xraw, neg, big);
+        solve<L, FWD, uint64_t, L>(Pc, Px, d.dt, xraw - Px[L], lw, i, o.makespan[dir],
+                                   o.bits[dir], o.nseg[dir], o.status[dir]);
+    }
+}
+
+template <int L, bool FWD>
+cudaError_t launch_fused_list(const GenParams &g, const GenTables *t, const FusedOut &o,
+                              cudaStream_t stream)
+{
+    using K64 = Small<L, uint64_t, L>;
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(fused_list_kernel<L, FWD>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             K64::kTableBytes);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    int64_t lgrid = (g.batch + 31) / 32;
+    if (lgrid > int64_t(sm_count()) * 4) lgrid = int64_t(sm_count()) * 4;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(unsigned(lgrid));
+    lc.blockDim = dim3(32);
+    lc.dynamicSmemBytes = K64::kTableBytes;
+    lc.stream = stream;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, fused_list_kernel<L, FWD>, g, t, o);
+}
+
+template <int L, bool FWD>
+cudaError_t launch_fused_dir(const GenParams &g, const GenTables *t, const FusedOut &o,
+                             cudaStream_t stream)
+{
+    using K32 = Small<L, uint32_t, kKeepCols>;
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        cudaError_t e = cudaFuncSetAttribute(fused_dense_kernel<L, FWD>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             K32::kWarpBytes);
+        if (e != cudaSuccess) return e;
+        int n = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fused_dense_kernel<L, FWD>, 32,
+                                                          K32::kWarpBytes);
+        if (e != cudaSuccess) return e;
+        per_sm = n > 0 ? n : 1;
+    }
+    const int64_t tiles = (g.batch + 31) / 32;
+    int64_t grid = int64_t(sm_count()) * per_sm;
+    if (grid > tiles) grid = tiles;
+    fused_dense_kernel<L, FWD><<<unsigned(grid), 32, K32::kWarpBytes, stream>>>(g, t, o);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return launch_fused_list<L, FWD>(g, t, o, stream);
+}
+
+template <int L>
+cudaError_t launch_fused_L(const GenParams &g, const GenTables *t, const FusedOut &o,
+                           cudaStream_t stream)
+{
+    cudaError_t e = launch_fused_dir<L, true>(g, t, o, stream);
+    if (e != cudaSuccess) return e;
+    return launch_fused_dir<L, false>(g, t, o, stream);
+}
+
+}  // namespace
+
+size_t fused_workspace_bytes(int64_t batch) { return fused_tables_offset(batch) + sizeof(GenTables); }
+
+// Generate-and-solve for 1 <= L <= 16: outputs [2][batch] (forward first).
+cudaError_t launch_fused(const GenParams &g, int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                         int32_t *status, void *workspace, cudaStream_t stream)
+{
+    const int64_t B = g.batch;
+    const int W = words_for(g.L);
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    FusedOut o;
+    for (int d = 0; d < 2; ++d) {
+        o.makespan[d] = makespan + d * B;
+        o.bits[d] = bits + d * B * W;
+        o.nseg[d] = nseg ? nseg + d * B : nullptr;
+        o.status[d] = status ? status + d * B : nullptr;
+        o.wide_count[d] = reinterpret_cast<uint32_t *>(ws) + d;
+        o.wide_list[d] = reinterpret_cast<uint32_t *>(ws + 256) + d * B;
+    }
+    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), stream);
+    if (e != cudaSuccess) return e;
+    GenTables *t = reinterpret_cast<GenTables *>(ws + fused_tables_offset(B));
+    copy_tables_kernel<<<1, 256, 0, stream>>>(g, t);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+#define DC_FUSED_CASE(LL) \
+    case LL: return launch_fused_L<LL>(g, t, o, stream);
+    switch (g.L) {
+        DC_FUSED_CASE(1) DC_FUSED_CASE(2) DC_FUSED_CASE(3) DC_FUSED_CASE(4)
+        DC_FUSED_CASE(5) DC_FUSED_CASE(6) DC_FUSED_CASE(7) DC_FUSED_CASE(8)
+        DC_FUSED_CASE(9) DC_FUSED_CASE(10) DC_FUSED_CASE(11) DC_FUSED_CASE(12)
+        DC_FUSED_CASE(13) DC_FUSED_CASE(14) DC_FUSED_CASE(15) DC_FUSED_CASE(16)
+        default: return cudaErrorInvalidValue;
+    }
+#undef DC_FUSED_CASE
+}
+
+}  // namespace dc

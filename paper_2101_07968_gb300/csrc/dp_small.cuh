@@ -1,0 +1,404 @@
+// Device building blocks of the short-L (1 <= L <= 16) DP, shared by the dense
+// and list passes (dp_small.cu) and the fused generate-and-solve passes
+// (dp_fused.cu). The design notes are at the top of dp_small.cu.
+#pragma once
+
+#include "gen_device.cuh"
+
+namespace dc {
+
+int sm_count();  // SMs of the current device (dp_small.cu)
+
+namespace {
+
+
+#ifndef DC_KEEP_COLS
+#define DC_KEEP_COLS 4
+#endif
+#ifndef DC_SMALL_MINB
+#define DC_SMALL_MINB 16  // resident single-warp CTAs per SM the registers must allow
+#endif
+#ifndef DC_TREE_MIN
+#define DC_TREE_MIN 1
+#endif
+constexpr int kTbGroup = 4;  // traceback candidates loaded per round
+constexpr int kKeepCols = DC_KEEP_COLS;  // the 32-bit pass stores columns 2..kKeepCols
+
+// index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
+__host__ __device__ constexpr int cell2(int L, int m, int n)
+{
+    return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
+}
+
+// Row stride of the staging buffer in int64 units: odd, so that the 16 lanes of a
+// half-warp reading 64-bit words of their own rows hit 16 distinct bank pairs.
+__host__ __device__ constexpr int stage_stride(int L) { return (L % 2 == 0) ? L + 1 : L; }
+
+// Stored columns 2..C with C = min(keep, L-1); KEEP = L keeps them all.
+template <int L, typename T, int KEEP>
+struct Small {
+    static constexpr int kLast = KEEP < L - 1 ? KEEP : L - 1;  // last stored column
+    static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
+    static constexpr int kOffS = kCells;                                // S[0..L]
+    static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
+    static constexpr int kLaneVals = kCells + 2 * (L + 1);
+    static constexpr int kStride = stage_stride(L);          // staging row stride (int64, odd)
+    static constexpr int kStageBytes = 2 * 32 * kStride * 8;   // comp + xfer rows of a tile
+    static constexpr int kTableBytes = 32 * kLaneVals * int(sizeof(T));
+    // staging and table share the warp's area
+    static constexpr int kWarpBytes = kStageBytes > kTableBytes ? kStageBytes : kTableBytes;
+};
+
+template <typename T>
+__device__ __forceinline__ T lds(const T *lane_base, int v) { return lane_base[32 * v]; }
+
+// The fill. lw = this lane's values in shared memory (value v at lw[32*v]).
+template <int L, bool FWD, typename T, int KEEP>
+__device__ __forceinline__ void fill(const T (&S)[L + 1], const T (&Rb)[L + 1], T dtv, T c,
+                                     T *lw, T &best_T, int &best_s)
+{
+    T col[L + 1];
+#pragma unroll
+    for (int m = 1; m <= L; ++m) col[m] = T((FWD ? T(dtv + Rb[m]) : Rb[m]) + S[m] + c);
+    best_T = col[L];
+    best_s = 1;
+#pragma unroll
+    for (int n = 2; n <= L; ++n) {
+        // rows in descending order so column n overwrites column n-1 in place:
+        // row m reads rows k < m, which still hold column n-1.
+#pragma unroll
+        for (int m = L; m >= n; --m) {
+            const T R = FWD ? T(T(n) * dtv + Rb[m]) : Rb[m];
+            constexpr int kMax = L;
+            T cand[kMax];
+            const int cnt = m - n + 1;  // k = n-1 .. m-1
+#pragma unroll
+            for (int j = 0; j < cnt; ++j) cand[j] = T(dmax(col[n - 1 + j], R) - S[n - 1 + j]);
+            if (DC_TREE_MIN) {  // balanced tree: log-depth chains
+#pragma unroll
+                for (int w = 1; w < cnt; w *= 2) {
+#pragma unroll
+                    for (int j = 0; j + w < cnt; j += 2 * w) cand[j] = dmin(cand[j], cand[j + w]);
+                }
+            } else {
+#pragma unroll
+                for (int j = 1; j < cnt; ++j) cand[0] = dmin(cand[0], cand[j]);
+            }
+            col[m] = T(cand[0] + S[m] + c);
+            if (n <= Small<L, T, KEEP>::kLast) lw[32 * cell2(L, m, n)] = col[m];
+        }
+        if (col[L] < best_T) {  // strict: the lowest n wins ties
+            best_T = col[L];
+            best_s = n;
+        }
+    }
+}
+
+// X[k][n-1] during the traceback: column 1 from S and R, others from the table.
+template <int L, bool FWD, typename T, int KEEP>
+__device__ __forceinline__ T prev_cell(const T *lw, int k, int nm1, T dtv, T c)
+{
+    using K = Small<L, T, KEEP>;
+    if (nm1 == 1) {
+        const T r = lds(lw, K::kOffR + k);
+        return T((FWD ? T(dtv + r) : r) + lds(lw, K::kOffS + k) + c);
+    }
+    return lds(lw, cell2(L, k, nm1));
+}
+
+// Solve one instance (row data already reduced to 64-bit prefix sums in
+// processing order) and write its outputs.
+// Returns false (writing nothing) when the optimum's traceback needs a column the
+// pass did not keep; the caller then lists the instance for the full pass.
+template <int L, bool FWD, typename T, int KEEP>
+__device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+                                      int64_t dti, uint64_t shift, T *lw, int64_t i,
+                                      int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                                      int32_t *status)
+{
+    using K = Small<L, T, KEEP>;
+    constexpr int W = (L - 1 + 31) / 32;
+    T S[L + 1], Rb[L + 1];
+#pragma unroll
+    for (int m = 0; m <= L; ++m) {
+        S[m] = T(FWD ? Pc[m] : Px[m]);
+        Rb[m] = T(FWD ? Px[m] : Pc[m]);
+        lw[32 * (K::kOffS + m)] = S[m];
+        lw[32 * (K::kOffR + m)] = Rb[m];
+    }
+    const T dtv = T(dti);
+    const T c = FWD ? T(0) : dtv;
+    T Tbest;
+    int s;
+    fill<L, FWD, T, KEEP>(S, Rb, dtv, c, lw, Tbest, s);
+    if (s - 1 > K::kLast && s - 1 >= 2) return false;
+
+    // traceback: from (L, s) step to the lowest k whose candidate equals the
+    // cell, set p_k / g_k, continue at (k, n-1)
+    uint32_t word = 0;
+    int err = 0;
+    int m = L, n = s;
+    T cell = Tbest;
+    while (n > 1) {
+        const T rm = lds(lw, K::kOffR + m);
+        const T R = FWD ? T(T(n) * dtv + rm) : rm;
+        const T target = T(cell - lds(lw, K::kOffS + m) - c);
+        // candidates in groups of kTbGroup: the loads issue back to back, then the
+        // compares run from the highest k down so that the lowest match wins
+        int k = -1;
+        T fk = T(0);
+        for (int k0 = n - 1; k0 < m && k < 0; k0 += kTbGroup) {
+            T f[kTbGroup], sk[kTbGroup];
+#pragma unroll
+            for (int u = 0; u < kTbGroup; ++u) {
+                const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
+                f[u] = prev_cell<L, FWD, T, KEEP>(lw, kk, n - 1, dtv, c);
+                sk[u] = lds(lw, K::kOffS + kk);
+            }
+#pragma unroll
+            for (int u = kTbGroup - 1; u >= 0; --u) {
+                if (k0 + u < m && T(dmax(f[u], R) - sk[u]) == target) {
+                    k = k0 + u;
+                    fk = f[u];
+                }
+            }
+        }
+        if (k < 0) {  // cannot happen: the fill and this check use the same arithmetic
+            err = 1;
+            break;
+        }
+        word |= 1u << ((k - 1) & 31);
+        m = k;
+        n -= 1;
+        cell = fk;
+    }
+    makespan[i] = int64_t(uint64_t(Tbest) + shift);
+    if (nseg) nseg[i] = s;
+    if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+    if (W > 0) bits[i * W] = word;
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// The 32-bit pass in shifted form. Every value is taken relative to the time
+// the last pull (forward) or push (backward) of its cell can start, which turns
+// a transition into one add-then-max and the minimum into 3-input mins: on
+// GB300 both are single integer-ALU instructions (the DPX forms), so a transition
+// costs 1.5 ALU-pipe instructions instead of 2.
+//
+// forward (P = transfer prefix, FC = compute prefix, G[k] = FC[L] - FC[k],
+// Q[m] = dt + P[m]): with B = X - n*dt - P[m] + G[m] (X as above) and
+// A[k] = B[k][n-1] + P[k] - dt,
+//   B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[m][1] = FC[L] + P[m],
+//   X[L][n] = B[L][n] + n*dt + P[L];
+// the next column's A[m] is that minimum less dt;
+// backward (BC = compute prefix, NGT[k] = -(transfer prefix)): with
+// E = X - n*dt - S[m],
+//   E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),  E[m][1] = BC[m],
+//   X[L][n] = E[L][n] + n*dt + S[L].
+// Both are min_k max(u[m] + V[k], C[k]) with a row constant u and the previous
+// column C in the max operand. Each candidate differs from Eq. 8/9's by a
+// constant of its row, so every argmin is the same. All values and sums lie in
+// [-2^31, 2^31) when the capped bound L*dt + sum(comp) + sum(capped xfer) is
+// below 2^31; other instances take the 64-bit pass. The table stores A (forward)
+// or E (backward) for columns 2..kKeepCols; the lane's two arrays hold U = Q and
+// V = G (forward) or U = BC and V = NGT.
+
+// Minimum of c[0..cnt-1] (cnt a compile-time constant after unrolling): two
+// chains of 3-input mins, so that each row has two independent dependency chains
+// and the rows of a column interleave.
+template <int N>
+__device__ __forceinline__ int32_t min_fold3(const int32_t (&c)[N], int cnt)
+{
+    if (cnt == 1) return c[0];
+    if (cnt == 2) return min(c[0], c[1]);
+    int32_t a = c[0], b = c[1];
+    int j = 2;
+#pragma unroll
+    for (; j + 3 < cnt; j += 4) {
+        a = __vimin3_s32(a, c[j], c[j + 1]);
+        b = __vimin3_s32(b, c[j + 2], c[j + 3]);
+    }
+    if (j + 1 < cnt) return __vimin3_s32(__vimin3_s32(a, b, c[j]), c[j + 1], cnt > j + 2 ? c[j + 2] : c[j + 1]);
+    if (j < cnt) return __vimin3_s32(a, b, c[j]);
+    return min(a, b);
+}
+
+template <int L, bool FWD>
+__device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
+                                       int32_t dt, int32_t fcL, int32_t *lw, int32_t &bestV,
+                                       int &best_s)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    // forward: U = Q, V = G, col = A; backward: U = BC, V = NGT, col = E
+    int32_t col[L + 1];
+#pragma unroll
+    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL + U[m] - dt : U[m];
+    bestV = (FWD ? fcL : U[L]) + dt;
+    best_s = 1;
+#pragma unroll
+    for (int n = 2; n <= L; ++n) {
+        int32_t last = 0;  // B[L][n] or E[L][n]
+#pragma unroll
+        for (int m = L; m >= n; --m) {  // descending: column n overwrites column n-1 in place
+            const int cnt = m - n + 1;  // k = n-1 .. m-1
+            const int32_t u = FWD ? U[m] : U[m] - (n - 1) * dt;
+            int32_t c[L];
+#pragma unroll
+            for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(u, V[n - 1 + j], col[n - 1 + j]);
+            const int32_t b = min_fold3<L>(c, cnt);
+            if (m == L) last = FWD ? b - U[L] : b;
+            col[m] = FWD ? b - dt : b;
+            if (n <= K::kLast) lw[32 * cell2(L, m, n)] = col[m];
+        }
+        const int32_t v = last + n * dt;
+        if (v < bestV) {  // strict: the lowest n wins ties
+            bestV = v;
+            best_s = n;
+        }
+    }
+}
+
+// The fill, the traceback and the outputs of one instance in shifted form.
+// Returns false (writing nothing) when the traceback needs a column the pass did
+// not keep.
+template <int L, bool FWD>
+__device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+                                        int64_t dti, uint64_t xraw, int32_t *lw, int64_t i,
+                                        int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                                        int32_t *status)
+{
+    using K = Small<L, uint32_t, kKeepCols>;
+    constexpr int W = (L - 1 + 31) / 32;
+    const int32_t dt = int32_t(dti);
+    const int32_t fcL = int32_t(Pc[L]);
+    int32_t U[L + 1], V[L + 1];
+#pragma unroll
+    for (int m = 0; m <= L; ++m) {
+        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]);
+        V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
+        lw[32 * (K::kOffR + m)] = U[m];
+        lw[32 * (K::kOffS + m)] = V[m];
+    }
+    int32_t bestV;
+    int s;
+    fill_e<L, FWD>(U, V, dt, fcL, lw, bestV, s);
+    if (s - 1 > K::kLast && s - 1 >= 2) return false;
+
+    // from (L, s) step to the lowest k whose candidate equals the cell, set
+    // p_k / g_k, continue at (k, n-1). A step compares every candidate at once
+    // (U and V still in registers, compile-time k): bit k of `hit` is set when
+    // candidate k equals the cell, and the lowest k inside [n-1, m-1] is the one
+    // Algorithm 3/4 keeps.
+    uint32_t word = 0;
+    int err = 0;
+    int m = L, n = s;
+    int32_t target = bestV - s * dt + (FWD ? U[L] : 0);  // B[L][s] + Q[L] or E[L][s]
+    while (n > 1) {
+        const int nm1 = n - 1;
+        const int32_t um = lds(lw, K::kOffR + m);
+        const int32_t u = FWD ? um : um - nm1 * dt;
+        uint32_t hit = 0u;
+        if (nm1 == 1) {  // column 1 is not stored: A = FC[L] + Q - dt, E = BC
+#pragma unroll
+            for (int k = 1; k < L; ++k) {
+                const int32_t f = FWD ? fcL + U[k] - dt : U[k];
+                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
+            }
+        } else {
+            const int base = cell2(L, 0, nm1);  // cell (k, n-1) is base + k
+#pragma unroll
+            for (int k = 1; k < L; ++k) {
+                const int32_t f = k >= nm1 ? lds(lw, base + k) : 0;
+                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
+            }
+        }
+        hit &= ((2u << (m - 1)) - 1u) & ~((1u << nm1) - 1u);  // k in [n-1, m-1]
+        if (hit == 0u) {  // cannot happen: the fill and this check use the same arithmetic
+            err = 1;
+            break;
+        }
+        const int k = __ffs(int(hit)) - 1;
+        word |= 1u << ((k - 1) & 31);
+        if (nm1 >= 2) {  // the cell (k, n-1): B + Q[k] = A + dt, or E
+            const int32_t fk = lds(lw, cell2(L, k, nm1));
+            target = FWD ? fk + dt : fk;
+        }
+        m = k;
+        n = nm1;
+    }
+    makespan[i] = int64_t(uint64_t(uint32_t(bestV)) + xraw);
+    if (nseg) nseg[i] = s;
+    if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
+    if (W > 0) bits[i * W] = word;
+    return true;
+}
+
+__device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
+{
+    const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
+
+// Issue the copies of tile `base` (rows base..base+rows-1) into the staging area.
+template <int L>
+__device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int64_t *comp,
+                                           const int64_t *xfer, int64_t base, int rows, int lane)
+{
+    constexpr int kStride = stage_stride(L);
+    const int64_t *gC = comp + base * L;
+    const int64_t *gX = xfer + base * L;
+    const int nel = rows * L;
+    for (int e = lane; e < nel; e += 32) {
+        const int r = e / L, cidx = e - r * L;
+        cp_async8(stC + r * kStride + cidx, gC + e);
+        cp_async8(stX + r * kStride + cidx, gX + e);
+    }
+    cp_async_commit();
+}
+
+// Read this lane's row (processing order) into 64-bit prefix sums; flag bad
+// input. Transfer costs are capped at the row's total compute: shifted by
+// n*dt + (transfer prefix), every DP value lies in [0, total compute] and the
+// recurrence sees transfer costs only through saturating differences, so the cap
+// changes no comparison (same decision) and lowers the makespan by exactly
+// sum(xfer) - sum(capped xfer), returned in `shift`.
+template <int L, bool FWD, typename Src>
+__device__ __forceinline__ void row_prefix(Src get, uint64_t (&Pc)[L + 1], uint64_t (&Px)[L + 1],
+                                           uint64_t &xraw, bool &neg, bool &big)
+{
+    uint64_t tc = 0;
+    xraw = 0;
+#pragma unroll
+    for (int r = 1; r <= L; ++r) {
+        int64_t cv, xv;
+        get(FWD ? r - 1 : L - r, cv, xv);
+        neg |= (cv < 0) | (xv < 0);
+        big |= ((cv | xv) >> 52) != 0;
+        tc += uint64_t(cv);
+        xraw += uint64_t(xv);
+    }
+    Pc[0] = 0;
+    Px[0] = 0;
+#pragma unroll
+    for (int r = 1; r <= L; ++r) {
+        int64_t cv, xv;
+        get(FWD ? r - 1 : L - r, cv, xv);
+        Pc[r] = Pc[r - 1] + uint64_t(cv);
+        Px[r] = Px[r - 1] + (uint64_t(xv) < tc ? uint64_t(xv) : tc);
+    }
+}
+
+__device__ __forceinline__ void write_failure(int st, int64_t i, int W, int64_t *makespan,
+                                              uint32_t *bits, int32_t *nseg, int32_t *status)
+{
+    makespan[i] = -int64_t(st);
+    if (nseg) nseg[i] = 0;
+    if (status) status[i] = st;
+    for (int w = 0; w < W; ++w) bits[i * W + w] = 0u;
+}
+
+}  // namespace
+}  // namespace dc

@@ -1,11 +1,10 @@
 // C ABI entry points (declared in include/dynacomm.h): host-side argument
 // checks, then kernel launches on the caller's stream. No allocation, no
 // synchronisation, no state kept between calls.
-#include "common.cuh"
+#include "gen_device.cuh"
 
 namespace dc {
 
-dc_status check_profile_cfg(const dc_profile_cfg *c);
 cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_t *bc,
                        int64_t *gt, int64_t *dt, cudaStream_t stream);
 
@@ -79,6 +78,32 @@ dc_status dc_profile_gen(const dc_profile_cfg *cfg, int64_t *fc, int64_t *pt, in
     if (cfg->batch == 0) return DC_OK;
     if (!fc || !pt || !bc || !gt || !dt) return DC_ERR_NULL;
     return dc::launch_gen(cfg, fc, pt, bc, gt, dt, stream) == cudaSuccess ? DC_OK : DC_ERR_CUDA;
+}
+
+size_t dc_schedule_generated_workspace_bytes(int64_t batch, int32_t L)
+{
+    if (batch < 0 || L < 1 || L > dc::kSmallLMax) return 0;
+    return dc::fused_workspace_bytes(batch);
+}
+
+dc_status dc_schedule_generated_batch(const dc_profile_cfg *cfg, int64_t *makespan,
+                                      uint32_t *bits, int32_t *nseg, int32_t *status,
+                                      void *workspace, size_t workspace_bytes,
+                                      cudaStream_t stream)
+{
+    if (!cfg) return DC_ERR_NULL;
+    const dc_status st = dc::check_profile_cfg(cfg);
+    if (st != DC_OK) return st;
+    if (cfg->L > dc::kSmallLMax || cfg->batch > int64_t(0xffffffffll)) return DC_ERR_BAD_SHAPE;
+    if (cfg->batch == 0) return DC_OK;
+    if (!makespan || (!bits && dc::words_for(cfg->L) > 0)) return DC_ERR_NULL;
+    if (!workspace || workspace_bytes < dc::fused_workspace_bytes(cfg->batch))
+        return DC_ERR_WORKSPACE;
+    static thread_local dc::GenParams g;  // 25 KB: kept off the caller's stack
+    dc::fill_gen_params(cfg, g);
+    return dc::launch_fused(g, makespan, bits, nseg, status, workspace, stream) == cudaSuccess
+               ? DC_OK
+               : DC_ERR_CUDA;
 }
 
 size_t dc_schedule_workspace_bytes(int64_t batch, int32_t L)

@@ -62,6 +62,9 @@ _SIGNATURES = {
     "dc_eval_timeline_batch": (_I32, [_I64, _I32, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_schedule_batch_static": (_I32, [_I32, _I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
                                         _VP]),
+    "dc_schedule_generated_workspace_bytes": (_SZ, [_I64, _I32]),
+    "dc_schedule_generated_batch": (_I32, [ctypes.POINTER(dc_profile_cfg), _VP, _VP, _VP, _VP,
+                                           _VP, _SZ, _VP]),
     "dc_greedy_forward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_greedy_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_status_string": (ctypes.c_char_p, [_I32]),
@@ -192,6 +195,19 @@ def dc_eval_timeline_batch(batch, L, direction, comp, xfer, dt, bits, makespan,
         _ptr(makespan), _stream(stream)))
 
 
+def dc_schedule_generated_workspace_bytes(batch: int, L: int) -> int:
+    return int(lib().dc_schedule_generated_workspace_bytes(int(batch), int(L)))
+
+
+def dc_schedule_generated_batch(cfg, makespan, bits, nseg, status, workspace, workspace_bytes,
+                                stream=None) -> int:
+    keep: list = []
+    c = cfg if isinstance(cfg, dc_profile_cfg) else make_cfg(cfg, keep)
+    return int(lib().dc_schedule_generated_batch(
+        ctypes.byref(c), _ptr(makespan), _ptr(bits), _ptr(nseg), _ptr(status), _ptr(workspace),
+        int(workspace_bytes), _stream(stream)))
+
+
 def dc_greedy_forward_batch(batch, L, fc, pt, dt, makespan, bits, stream=None) -> int:
     return int(lib().dc_greedy_forward_batch(int(batch), int(L), _ptr(fc), _ptr(pt), _ptr(dt),
                                              _ptr(makespan), _ptr(bits), _stream(stream)))
@@ -264,6 +280,35 @@ def eval_timeline(direction: int, comp, xfer, dt, bits, stream=None):
     _check(dc_eval_timeline_batch(B, L, direction, comp, xfer, dt, bits, out, stream),
            "dc_eval_timeline_batch")
     return out
+
+
+class GeneratedScheduler:
+    """Generate-and-solve (L <= 16) for a config dict with fixed batch and L:
+    both directions without materialising the profiles. run() returns dict of
+    makespan [2, B] int64, bits [2, B, max(W,1)] int32 view, nseg and status
+    [2, B] int32 (index 0 forward, 1 backward)."""
+
+    def __init__(self, cfg: dict, device="cuda"):
+        import torch
+        self.cfg, self.keep = cfg, []
+        self.c = make_cfg(cfg, self.keep)
+        B, L = int(cfg["batch"]), int(cfg["L"])
+        self.W = words(L)
+        self.ws_bytes = dc_schedule_generated_workspace_bytes(B, L)
+        if self.ws_bytes == 0:
+            raise DynaCommError(DC_ERR_BAD_SHAPE, "dc_schedule_generated_workspace_bytes")
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.out = {"makespan": torch.empty((2, B), dtype=torch.int64, device=device),
+                    "bits": torch.empty((2, B, max(self.W, 1)), dtype=torch.int32, device=device),
+                    "nseg": torch.empty((2, B), dtype=torch.int32, device=device),
+                    "status": torch.empty((2, B), dtype=torch.int32, device=device)}
+
+    def run(self, stream=None) -> dict:
+        o = self.out
+        _check(dc_schedule_generated_batch(self.c, o["makespan"], o["bits"], o["nseg"],
+                                           o["status"], self.ws, self.ws_bytes, stream),
+               "dc_schedule_generated_batch")
+        return o
 
 
 def greedy(direction: int, comp, xfer, dt, stream=None) -> dict:
