@@ -329,13 +329,26 @@ __device__ __forceinline__ void fill_tiles_s32(int L, int n, int32_t ndt1, const
         }
         const int kf = k1 < bot ? k1 : bot;  // k < bot: every row of the block takes it
         int k = k0;
-        for (; k + 1 < kf; k += 2) {
-            const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
-            const int32_t c1 = prev[skew(k + 1)], v1 = V[skew(k + 1)];
+        while (k + 1 < kf) {
+            // pairs inside the 32-aligned block of k, where skew(k) is linear in k
+            const int kend = min(kf, (k | 31) + 1);
+            const int32_t *pc = prev + skew(k), *pv = V + skew(k);
+            for (; k + 1 < kend; k += 2, pc += 2, pv += 2) {
+                const int32_t c0 = pc[0], v0 = pv[0], c1 = pc[1], v1 = pv[1];
 #pragma unroll
-            for (int jj = 0; jj < kRB; ++jj)
-                acc[jj] = __vimin3_s32(acc[jj], cand_s32(c0, Ur[jj], v0),
-                                       cand_s32(c1, Ur[jj], v1));
+                for (int jj = 0; jj < kRB; ++jj)
+                    acc[jj] = __vimin3_s32(acc[jj], cand_s32(c0, Ur[jj], v0),
+                                           cand_s32(c1, Ur[jj], v1));
+            }
+            if (k + 1 == kend && kend < kf) {  // a pair across the block boundary
+                const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
+                const int32_t c1 = prev[skew(k + 1)], v1 = V[skew(k + 1)];
+#pragma unroll
+                for (int jj = 0; jj < kRB; ++jj)
+                    acc[jj] = __vimin3_s32(acc[jj], cand_s32(c0, Ur[jj], v0),
+                                           cand_s32(c1, Ur[jj], v1));
+                k += 2;
+            }
         }
         if (k < kf) {
             const int32_t c0 = prev[skew(k)], v0 = V[skew(k)];
@@ -640,10 +653,11 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
 //   E[m][n] + G[m] = min_{k} max(A[k] - Q[m], G[k]),  E[m][1] = FC[m].
 // A[k] and Q[m] are large but only a non-negative difference below 2^30 matters,
 // so inside a tile both are taken relative to P at the tile's lowest row: when
-// the tile's rows span less than 2^30 of transfer, A - P[bot] clamped below at
-// -2^30 and Q - P[bot] are signed 32-bit and the transition is one add-then-max
-// (two candidates folding with one 3-input min); other tiles use the same
-// formula in 64-bit. Candidates differ from Eq. 8's
+// the tile's rows span less than 2^30 of transfer, Q - P[bot] is signed 32-bit,
+// the candidates of the far k (P[k] more than 2^30 below P[bot]) reduce to their
+// G, and for the others A - P[bot] is signed 32-bit: a transition is one
+// add-then-max (two candidates folding with one 3-input min); other tiles use
+// the same formula in 64-bit. Candidates differ from Eq. 8's
 // by the row constant n*dt + P[m] + G[m]: every argmin is unchanged, and
 // F[L][n] = E[L][n] + n*dt + P[L]. Needs FC[L] < 2^29.
 constexpr int32_t kSpan = 1 << 30;
@@ -671,11 +685,27 @@ __device__ __forceinline__ void fill_tiles_efwd(int L, int n, uint64_t dtv, cons
                 const int m = bot + jj <= top ? bot + jj : top;
                 NQr[jj] = -int32_t(dtv + (P[skew(m)] - base));
             }
-            auto rel = [&](int k) {  // A[k] - base, clamped below at -2^30
-                const int64_t ad = int64_t(A[skew(k)] - base);
-                return ad < -int64_t(kSpan) ? -kSpan : int32_t(ad);
-            };
-            int k = k0;
+            // k with P[k] < base - 2^30 have A[k] - base < -2^30 + FC[L] < -2^29 (A[k]
+            // <= P[k] + FC[L]), so their candidate is exactly G[k]; G is non-increasing,
+            // so together they contribute G at the last of them. The others have
+            // A[k] - base in [-2^30, 2^30 + 2^29): the low 32-bit words' difference.
+            int lo = k0, hi = kf;  // P is non-decreasing: the first k past the far ones
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (P[skew(mid)] + uint64_t(kSpan) < base)
+                    lo = mid + 1;
+                else
+                    hi = mid;
+            }
+            if (lo > k0) {
+                const int32_t gfar = G[skew(lo - 1)];
+#pragma unroll
+                for (int jj = 0; jj < kRB; ++jj) acc[jj] = min(acc[jj], gfar);
+            }
+            const uint32_t *Alo = reinterpret_cast<const uint32_t *>(A);  // low words
+            const uint32_t blo = uint32_t(base);
+            auto rel = [&](int k) { return int32_t(Alo[2 * skew(k)] - blo); };
+            int k = lo;
             for (; k + 1 < kf; k += 2) {
                 const int32_t a0 = rel(k), g0 = G[skew(k)];
                 const int32_t a1 = rel(k + 1), g1 = G[skew(k + 1)];
