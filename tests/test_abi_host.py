@@ -125,3 +125,34 @@ def test_binding_refuses_host_tensors(lib):
     import torch
     with pytest.raises(ValueError):
         dc._ptr(torch.zeros(3, dtype=torch.int64))
+
+
+@pytest.mark.parametrize("fn", ["dc_greedy_forward_batch", "dc_greedy_backward_batch"])
+def test_greedy_host_checks(lib, fn):
+    f = getattr(dc, fn)
+    assert f(5, 0, FAKE, FAKE, FAKE, FAKE, FAKE) == dc.DC_ERR_BAD_SHAPE
+    assert f(5, 4097, FAKE, FAKE, FAKE, FAKE, FAKE) == dc.DC_ERR_BAD_SHAPE
+    assert f(-1, 8, FAKE, FAKE, FAKE, FAKE, FAKE) == dc.DC_ERR_BAD_SHAPE
+    assert f(2**32, 8, FAKE, FAKE, FAKE, FAKE, FAKE) == dc.DC_ERR_BAD_SHAPE
+    assert f(0, 8, None, None, None, None, None) == dc.DC_OK
+    assert f(5, 8, None, FAKE, FAKE, FAKE, FAKE) == dc.DC_ERR_NULL
+    assert f(5, 8, FAKE, FAKE, FAKE, None, FAKE) == dc.DC_ERR_NULL
+    assert f(5, 8, FAKE, FAKE, FAKE, FAKE, None) == dc.DC_ERR_NULL
+
+
+def test_generated_host_checks(lib):
+    f = dc.dc_schedule_generated_batch
+    q = dc.dc_schedule_generated_workspace_bytes
+    assert q(1000, 16) >= 256 + 8 * 1000 and q(1000, 17) == 0 and q(-1, 8) == 0 and q(5, 0) == 0
+    cfg = wl.with_batch(wl.config("vgg16"), 1000)
+    need = q(1000, 16)
+    bad = dict(cfg)
+    bad["rate_lo"] = 0
+    assert f(bad, FAKE, FAKE, None, None, FAKE, need) == dc.DC_ERR_BAD_CONFIG
+    deep = wl.with_batch(wl.config("deepchain"), 10)
+    assert f(deep, FAKE, FAKE, None, None, FAKE, 1 << 30) == dc.DC_ERR_BAD_SHAPE
+    assert f(wl.with_batch(cfg, 0), None, None, None, None, None, 0) == dc.DC_OK
+    assert f(cfg, None, FAKE, None, None, FAKE, need) == dc.DC_ERR_NULL
+    assert f(cfg, FAKE, None, None, None, FAKE, need) == dc.DC_ERR_NULL
+    assert f(cfg, FAKE, FAKE, None, None, None, need) == dc.DC_ERR_WORKSPACE
+    assert f(cfg, FAKE, FAKE, None, None, FAKE, need - 1) == dc.DC_ERR_WORKSPACE
