@@ -129,7 +129,8 @@ def load_json(path):
 def dp_source_hash() -> str:
     import hashlib
     h = hashlib.sha256()
-    for name in ("dp_small.cu", "dp_mid.cu", "dp_group.cu", "common.cuh", "dynacomm_abi.cu"):
+    for name in ("dp_small.cu", "dp_small.cuh", "dp_mid.cu", "dp_group.cu", "common.cuh",
+                 "dynacomm_abi.cu"):
         with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
