@@ -2,19 +2,25 @@
 // Eq. 9 / Algorithm 4), in 32-bit or 64-bit arithmetic per instance.
 //
 // Used for L > 64, and for the instances the thread-per-instance kernels list
-// (64-bit values, or a traceback deeper than they keep). Transfer costs are
-// capped at the total compute first (exact; see the short-L kernel).
+// (values beyond their 32-bit form, or a traceback deeper than they keep).
+// Transfer costs are capped at the total compute first (exact; see the short-L
+// kernel).
 //
 // Same processing-order template as the small kernel:
 //   X[m][n] = min_{k in [n-1, m-1]} max(X[k][n-1], R(m,n)) - S[k] + S[m] + c.
-// Column n's (row block, k chunk) tiles are spread over the CTA's threads (8 rows
-// x up to 64 candidates per tile, register-blocked), partial row minima are
-// combined with shared-memory atomicMin, then the column is finalised; columns
-// run in sequence with CTA barriers between them. Every finished cell is also
-// written to the instance's DP table (shared memory for L <= 64, otherwise a
-// per-CTA slot of the caller's workspace). After the fill, warp 0 picks the lowest n minimising X[L][n] and
-// walks the traceback, finding each Path[m][n] (the lowest k whose candidate
-// equals the cell) with one ballot per 32 candidates.
+// Per instance, the arithmetic is the first that is exact: the shifted signed
+// 32-bit form of the short kernels (capped bound below 2^31), the shifted forms
+// of this file for wider instances (backward with total compute below 2^31,
+// forward below 2^29), the literal template in 32 bits (bound below 2^32), else
+// in 64 bits. Column n's (row block, k chunk) tiles are spread over the CTA's
+// threads (8 rows x up to 64 candidates per tile, register-blocked), partial row
+// minima are combined with shared-memory atomicMin, then the column is
+// finalised; columns run in sequence with CTA barriers between them. Every
+// finished cell is also written to the instance's DP table (shared memory for
+// L <= 64, otherwise a per-CTA slot of the caller's workspace). After the fill,
+// warp 0 picks the lowest n minimising X[L][n] and walks the traceback, finding
+// each Path[m][n] (the lowest k whose candidate equals the cell) with one ballot
+// per 32 candidates.
 #include "common.cuh"
 
 namespace dc {

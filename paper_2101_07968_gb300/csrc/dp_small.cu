@@ -11,22 +11,24 @@
 // Design (GB300):
 //  * one instance per thread, 32 instances per warp, no inter-thread traffic in
 //    the fill; the DP column lives in registers with compile-time indices;
-//  * the fill keeps only the minimum VALUE per cell (max, subtract, min per
-//    transition: two integer-ALU-pipe operations, the subtraction can issue on
-//    the FMA pipe). Finished cells go to the lane's slice of shared memory; the
-//    traceback recovers Path[m][n] as the lowest k whose candidate equals the
-//    cell, which is the k Algorithm 3/4 keeps with its strict-improvement test.
-//    Column 1 (X[m][1] = R(m,1) + S[m] + c) and column L (one cell, the
-//    makespan) are not stored. The 32-bit pass stores only columns 2..kKeepCols:
-//    the traceback of an s-segment optimum reads columns 1..s-1 only, and s is
-//    small in practice (2-4 on CNN-shaped profiles); an instance whose s needs a
-//    deeper column is re-solved by the 64-bit pass, which keeps every column;
+//  * the 32-bit pass solves the shifted form (see the block before fill_e in
+//    dp_small.cuh): a transition is one add-then-max and two candidates fold
+//    into one 3-input min, 1.5 integer-ALU instructions on GB300;
+//  * the fill keeps only the minimum VALUE per cell; the traceback recovers
+//    Path[m][n] as the lowest k whose candidate equals the cell, which is the k
+//    Algorithm 3/4 keeps with its strict-improvement test. A step compares all
+//    of its candidates at once (bit mask, lowest set bit). Column 1 is derived,
+//    not stored, and the pass stores only columns 2..kKeepCols: the traceback of
+//    an s-segment optimum reads columns 1..s-1 only, and s is small in practice
+//    (2-5 on CNN-shaped profiles); an instance whose s needs a deeper column is
+//    re-solved by the 64-bit pass, which keeps every column;
 //  * transfer costs are first capped at the instance's total compute, which
-//    changes no decision (see row_prefix); 32-bit values whenever the capped
-//    bound L*dt + sum(capped xfer) + sum(comp) is below 2^32 - 1: every DP value
-//    and candidate lies in [0, bound], so the 32-bit fill is exact. Other
-//    instances (and the deep ones above) are appended to a work list that a
-//    64-bit instantiation solves afterwards;
+//    changes no decision (see row_prefix); the shifted 32-bit form is exact
+//    whenever the capped bound L*dt + sum(capped xfer) + sum(comp) is below
+//    2^31. Other instances (and the deep ones above) are appended to a work list
+//    that a 64-bit instantiation of the literal template solves afterwards; that
+//    pass is launched early and waits in hardware for this one (programmatic
+//    dependent launch);
 //  * persistent warps: each warp walks 32-instance tiles. A tile's rows arrive
 //    by cp.async (coalesced 8-byte copies) in the warp's own table area, with
 //    an odd row stride so that every lane reads its own row without bank
