@@ -127,12 +127,17 @@ def load_json(path):
 
 
 def dp_source_hash() -> str:
+    """Hash of the DP sources' code (comments and blank space removed), which a
+    traffic record must match to be reported."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for name in ("dp_small.cu", "dp_small.cuh", "dp_mid.cu", "dp_group.cu", "common.cuh",
                  "dynacomm_abi.cu"):
-        with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name)) as f:
+            code = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
+        code = re.sub(r"//[^\n]*", "", code)
+        h.update("".join(code.split()).encode())
     return h.hexdigest()[:16]
 
 
