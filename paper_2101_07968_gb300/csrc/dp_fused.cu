@@ -65,27 +65,17 @@ __device__ __forceinline__ void fused_direction(const GenParams &g, const GenTab
         }
     }
     const int64_t dti = active ? d.dt : 0;
-    uint64_t Pc[L + 1], Px[L + 1], xraw;
-    bool neg = dti < 0, big = (dti >> 52) != 0;
-    row_prefix<L, FWD>(
-        [&](int col, int64_t &cv, int64_t &xv) {
-            cv = active ? stC[lane * K::kStride + col] : 0;
-            xv = active ? stX[lane * K::kStride + col] : 0;
-        },
-        Pc, Px, xraw, neg, big);
+    int32_t U[L + 1], V[L + 1];
+    uint64_t xraw;
+    bool wide;
+    int st;
+    row_uv<L, FWD>(stC + lane * K::kStride, stX + lane * K::kStride, dti, U, V, xraw, wide, st);
     __syncwarp();  // rows read: the lanes' table slices may be written
     if (!active) return;
-    int st = DC_OK;
-    if (neg)
-        st = DC_ERR_NEGATIVE;
-    else if (big || uint64_t(L) * uint64_t(dti) + Pc[L] + xraw >= uint64_t(kRangeLimit))
-        st = DC_ERR_RANGE;
-    const uint64_t bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];  // capped
     if (st != DC_OK) {
         write_failure(st, i, W, o.makespan[dir], o.bits[dir], o.nseg[dir], o.status[dir]);
-    } else if (bound > kShiftedLimit ||
-               !solve_e<L, FWD>(Pc, Px, dti, xraw, lw, i, o.makespan[dir], o.bits[dir],
-                                o.nseg[dir], o.status[dir])) {
+    } else if (wide || !solve_uv<L, FWD>(U, V, int32_t(dti), xraw, lw, i, o.makespan[dir],
+                                         o.bits[dir], o.nseg[dir], o.status[dir])) {
         o.wide_list[dir][atomicAdd(o.wide_count[dir], 1u)] = uint32_t(i);
     }
 }

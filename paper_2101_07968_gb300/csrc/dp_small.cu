@@ -17,11 +17,16 @@
 //  * the fill keeps only the minimum VALUE per cell; the traceback recovers
 //    Path[m][n] as the lowest k whose candidate equals the cell, which is the k
 //    Algorithm 3/4 keeps with its strict-improvement test. A step compares all
-//    of its candidates at once (bit mask, lowest set bit). Column 1 is derived,
-//    not stored, and the pass stores only columns 2..kKeepCols: the traceback of
-//    an s-segment optimum reads columns 1..s-1 only, and s is small in practice
-//    (2-5 on CNN-shaped profiles); an instance whose s needs a deeper column is
-//    re-solved by the 64-bit pass, which keeps every column;
+//    of its candidates at once (bit mask, lowest set bit), and every step runs
+//    the same code (column 1 is stored like the others), so the lanes of a warp
+//    at different depths do not split into separate paths. The pass stores only
+//    columns 1..kKeepCols: the traceback of an s-segment optimum reads columns
+//    1..s-1 only, and s is small in practice (2-5 on CNN-shaped profiles); an
+//    instance whose s needs a deeper column is re-solved by the 64-bit pass,
+//    which keeps every column;
+//  * a row whose costs all fit 32 bits (compute below 2^31 / L) gets its prefix
+//    sums in 32-bit arithmetic (fast_uv); other rows take the 64-bit prefix,
+//    which also classifies bad input;
 //  * transfer costs are first capped at the instance's total compute, which
 //    changes no decision (see row_prefix); the shifted 32-bit form is exact
 //    whenever the capped bound L*dt + sum(capped xfer) + sum(comp) is below
@@ -74,26 +79,18 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         const int64_t dti = active ? __ldg(dt + i) : 0;
         cp_async_wait_all();
         __syncwarp();
-        uint64_t Pc[L + 1], Px[L + 1], xraw;
-        bool neg = dti < 0, big = (dti >> 52) != 0;
-        row_prefix<L, FWD>(
-            [&](int col, int64_t &cv, int64_t &xv) {
-                cv = active ? stC[lane * K::kStride + col] : 0;
-                xv = active ? stX[lane * K::kStride + col] : 0;
-            },
-            Pc, Px, xraw, neg, big);
+        const int64_t *rc = stC + lane * K::kStride, *rx = stX + lane * K::kStride;
+        int32_t U[L + 1], V[L + 1];
+        uint64_t xraw;
+        bool wide;
+        int st;
+        row_uv<L, FWD>(rc, rx, dti, U, V, xraw, wide, st);
         __syncwarp();  // rows read: the lanes' table slices may be written
         if (!active) continue;
-        int st = DC_OK;
-        if (neg)
-            st = DC_ERR_NEGATIVE;
-        else if (big || uint64_t(L) * uint64_t(dti) + Pc[L] + xraw >= uint64_t(kRangeLimit))
-            st = DC_ERR_RANGE;
-        const uint64_t bound = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L];  // capped
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
-        } else if (bound > kShiftedLimit ||
-                   !solve_e<L, FWD>(Pc, Px, dti, xraw, lw, i, makespan, bits, nseg, status)) {
+        } else if (wide ||
+                   !solve_uv<L, FWD>(U, V, int32_t(dti), xraw, lw, i, makespan, bits, nseg, status)) {
             // 64-bit values, or a traceback deeper than the kept columns: work list
             wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
         }

@@ -39,7 +39,8 @@ template <int L, typename T, int KEEP>
 struct Small {
     static constexpr int kLast = KEEP < L - 1 ? KEEP : L - 1;  // last stored column
     static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
-    static constexpr int kOffS = kCells;                                // S[0..L]
+    static constexpr int kOffS = kCells;   // S[0..L] (64-bit pass)
+    static constexpr int kOffC1 = kCells;  // column 1, rows 1..L-1 (32-bit pass)
     static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
     static constexpr int kLaneVals = kCells + 2 * (L + 1);
     static constexpr int kStride = stage_stride(L);          // staging row stride (int64, odd)
@@ -201,8 +202,8 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
 // constant of its row, so every argmin is the same. All values and sums lie in
 // [-2^31, 2^31) when the capped bound L*dt + sum(comp) + sum(capped xfer) is
 // below 2^31; other instances take the 64-bit pass. The table stores A (forward)
-// or E (backward) for columns 2..kKeepCols; the lane's two arrays hold U = Q and
-// V = G (forward) or U = BC and V = NGT.
+// or E (backward) for columns 1..kKeepCols and the row U (U = Q forward, BC
+// backward); V (G forward, NGT backward) stays in registers.
 
 // Minimum of c[0..cnt-1] (cnt a compile-time constant after unrolling): two
 // chains of 3-input mins, so that each row has two independent dependency chains
@@ -233,7 +234,10 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
     // forward: U = Q, V = G, col = A; backward: U = BC, V = NGT, col = E
     int32_t col[L + 1];
 #pragma unroll
-    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL + U[m] - dt : U[m];
+    for (int m = 1; m <= L; ++m) {
+        col[m] = FWD ? fcL + U[m] - dt : U[m];
+        if (m < L) lw[32 * (K::kOffC1 + m)] = col[m];  // for the traceback
+    }
     bestV = (FWD ? fcL : U[L]) + dt;
     best_s = 1;
 #pragma unroll
@@ -259,27 +263,22 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
     }
 }
 
-// The fill, the traceback and the outputs of one instance in shifted form.
-// Returns false (writing nothing) when the traceback needs a column the pass did
-// not keep.
+// The fill, the traceback and the outputs of one instance in shifted form, from
+// its U and V rows (forward: U = dt + capped transfer prefix, V = FC[L] - compute
+// prefix; backward: U = compute prefix, V = -capped transfer prefix) and the raw
+// transfer sum. Returns false (writing nothing) when the traceback needs a column
+// the pass did not keep.
 template <int L, bool FWD>
-__device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
-                                        int64_t dti, uint64_t xraw, int32_t *lw, int64_t i,
-                                        int64_t *makespan, uint32_t *bits, int32_t *nseg,
-                                        int32_t *status)
+__device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
+                                         int32_t dt, uint64_t xraw, int32_t *lw, int64_t i,
+                                         int64_t *makespan, uint32_t *bits, int32_t *nseg,
+                                         int32_t *status)
 {
     using K = Small<L, uint32_t, kKeepCols>;
     constexpr int W = (L - 1 + 31) / 32;
-    const int32_t dt = int32_t(dti);
-    const int32_t fcL = int32_t(Pc[L]);
-    int32_t U[L + 1], V[L + 1];
+    const int32_t fcL = V[0];  // forward: FC[L]
 #pragma unroll
-    for (int m = 0; m <= L; ++m) {
-        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]);
-        V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
-        lw[32 * (K::kOffR + m)] = U[m];
-        lw[32 * (K::kOffS + m)] = V[m];
-    }
+    for (int m = 0; m <= L; ++m) lw[32 * (K::kOffR + m)] = U[m];  // the traceback reads U[m]
     int32_t bestV;
     int s;
     fill_e<L, FWD>(U, V, dt, fcL, lw, bestV, s);
@@ -298,20 +297,13 @@ __device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint6
         const int nm1 = n - 1;
         const int32_t um = lds(lw, K::kOffR + m);
         const int32_t u = FWD ? um : um - nm1 * dt;
+        // cell (k, n-1) is base + k; column 1 has its own row of the table
+        const int base = nm1 == 1 ? K::kOffC1 : cell2(L, 0, nm1);
         uint32_t hit = 0u;
-        if (nm1 == 1) {  // column 1 is not stored: A = FC[L] + Q - dt, E = BC
 #pragma unroll
-            for (int k = 1; k < L; ++k) {
-                const int32_t f = FWD ? fcL + U[k] - dt : U[k];
-                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
-            }
-        } else {
-            const int base = cell2(L, 0, nm1);  // cell (k, n-1) is base + k
-#pragma unroll
-            for (int k = 1; k < L; ++k) {
-                const int32_t f = k >= nm1 ? lds(lw, base + k) : 0;
-                if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
-            }
+        for (int k = 1; k < L; ++k) {
+            const int32_t f = k >= nm1 ? lds(lw, base + k) : 0;
+            if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
         }
         hit &= ((2u << (m - 1)) - 1u) & ~((1u << nm1) - 1u);  // k in [n-1, m-1]
         if (hit == 0u) {  // cannot happen: the fill and this check use the same arithmetic
@@ -320,10 +312,8 @@ __device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint6
         }
         const int k = __ffs(int(hit)) - 1;
         word |= 1u << ((k - 1) & 31);
-        if (nm1 >= 2) {  // the cell (k, n-1): B + Q[k] = A + dt, or E
-            const int32_t fk = lds(lw, cell2(L, k, nm1));
-            target = FWD ? fk + dt : fk;
-        }
+        const int32_t fk = lds(lw, base + k);  // the cell (k, n-1): B + Q[k] = A + dt, or E
+        target = FWD ? fk + dt : fk;
         m = k;
         n = nm1;
     }
@@ -331,6 +321,74 @@ __device__ __forceinline__ bool solve_e(const uint64_t (&Pc)[L + 1], const uint6
     if (nseg) nseg[i] = s;
     if (status) status[i] = err ? DC_ERR_INTERNAL : DC_OK;
     if (W > 0) bits[i * W] = word;
+    return true;
+}
+
+// U and V from 64-bit prefix sums (the caller has checked the 32-bit range).
+template <int L, bool FWD>
+__device__ __forceinline__ void shifted_uv(const uint64_t (&Pc)[L + 1], const uint64_t (&Px)[L + 1],
+                                           int64_t dti, int32_t (&U)[L + 1], int32_t (&V)[L + 1])
+{
+    const int32_t dt = int32_t(dti);
+    const int32_t fcL = int32_t(Pc[L]);
+#pragma unroll
+    for (int m = 0; m <= L; ++m) {
+        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]);
+        V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
+    }
+}
+
+__host__ __device__ constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2); }
+
+// The row's U and V in 32-bit arithmetic, for the common row whose costs all lie
+// in [0, 2^32) with every compute cost below 2^31 / L (then every compute sum is
+// exact in 32 bits) and dt below 2^31. rc, rx: the row's costs in layer order.
+// Returns false, computing nothing, for any other row: the caller takes the
+// 64-bit route (which also classifies negative and out-of-range input). On true,
+// `wide` says whether the capped bound L*dt + sum(comp) + sum(capped xfer) exceeds
+// the shifted form's limit. Transfers are capped at the total compute as in
+// row_prefix; the sums of capped transfers and raw transfers are kept in 64 bits.
+template <int L, bool FWD>
+__device__ __forceinline__ bool fast_uv(const int64_t *rc, const int64_t *rx, int64_t dti,
+                                        int32_t (&U)[L + 1], int32_t (&V)[L + 1], uint64_t &xraw,
+                                        bool &wide)
+{
+    constexpr int kCompBits = 31 - ceil_log2(L);
+    uint32_t cl[L], xl[L];
+    uint32_t hor = uint32_t(uint64_t(dti) >> 31), cor = 0u, tc = 0u;
+#pragma unroll
+    for (int r = 0; r < L; ++r) {
+        const int col = FWD ? r : L - 1 - r;
+        const uint2 c = *reinterpret_cast<const uint2 *>(rc + col);
+        const uint2 x = *reinterpret_cast<const uint2 *>(rx + col);
+        cl[r] = c.x;
+        xl[r] = x.x;
+        hor |= c.y | x.y;
+        cor |= c.x;
+        tc += c.x;
+    }
+    if ((hor | (cor >> kCompBits)) != 0u) return false;
+    uint32_t u = FWD ? uint32_t(dti) : 0u, v = FWD ? tc : 0u;
+    U[0] = int32_t(u);
+    V[0] = int32_t(v);
+    uint64_t px = 0, xr = 0;
+#pragma unroll
+    for (int r = 0; r < L; ++r) {
+        const uint32_t xc = min(xl[r], tc);
+        px += xc;
+        xr += xl[r];
+        if (FWD) {
+            u += xc;
+            v -= cl[r];
+        } else {
+            u += cl[r];
+            v -= xc;
+        }
+        U[r + 1] = int32_t(u);
+        V[r + 1] = int32_t(v);
+    }
+    xraw = xr;
+    wide = uint64_t(L) * uint64_t(dti) + tc + px > uint64_t(kShiftedLimit);
     return true;
 }
 
@@ -389,6 +447,33 @@ __device__ __forceinline__ void row_prefix(Src get, uint64_t (&Pc)[L + 1], uint6
         Pc[r] = Pc[r - 1] + uint64_t(cv);
         Px[r] = Px[r - 1] + (uint64_t(xv) < tc ? uint64_t(xv) : tc);
     }
+}
+
+// A staged row (rc, rx: its costs in layer order) to the 32-bit pass's U and V:
+// fast_uv when the row fits, else 64-bit prefix sums with the input checks.
+// st: DC_OK or the row's error; wide: the capped bound exceeds the shifted form's
+// limit (the instance belongs to the 64-bit pass).
+template <int L, bool FWD>
+__device__ __forceinline__ void row_uv(const int64_t *rc, const int64_t *rx, int64_t dti,
+                                       int32_t (&U)[L + 1], int32_t (&V)[L + 1], uint64_t &xraw,
+                                       bool &wide, int &st)
+{
+    st = DC_OK;
+    if (fast_uv<L, FWD>(rc, rx, dti, U, V, xraw, wide)) return;
+    uint64_t Pc[L + 1], Px[L + 1];
+    bool neg = dti < 0, big = (dti >> 52) != 0;
+    row_prefix<L, FWD>(
+        [&](int col, int64_t &cv, int64_t &xv) {
+            cv = rc[col];
+            xv = rx[col];
+        },
+        Pc, Px, xraw, neg, big);
+    if (neg)
+        st = DC_ERR_NEGATIVE;
+    else if (big || uint64_t(L) * uint64_t(dti) + Pc[L] + xraw >= uint64_t(kRangeLimit))
+        st = DC_ERR_RANGE;
+    wide = uint64_t(L) * uint64_t(dti) + Pc[L] + Px[L] > kShiftedLimit;  // capped bound
+    shifted_uv<L, FWD>(Pc, Px, dti, U, V);
 }
 
 __device__ __forceinline__ void write_failure(int st, int64_t i, int W, int64_t *makespan,
