@@ -35,13 +35,14 @@
 //    pass is launched early and waits in hardware for this one (programmatic
 //    dependent launch);
 //  * persistent warps: each warp walks 32-instance tiles. A tile's rows arrive
-//    by cp.async (coalesced 8-byte copies) in the warp's own table area, with
-//    an odd row stride so that every lane reads its own row without bank
-//    conflicts; the prefix sums then leave them in registers and the table
-//    overwrites them. Sharing the area keeps a warp at the table's size of
-//    shared memory, so 16 warps fit on an SM (the register limit at <= 128
-//    registers): more resident warps hide more latency than a separate
-//    prefetch buffer would.
+//    by cp.async (coalesced 16-byte copies of cost pairs for even L) in the
+//    warp's own table area, with a row stride at which every lane reads its own
+//    row without bank conflicts (stage_stride); the prefix sums then leave them
+//    in registers and the table overwrites them. Sharing the area keeps a warp
+//    at the table's size of shared memory, so 20 warps fit on an SM (the
+//    register limit at <= 96 registers): more resident warps hide more latency
+//    than a separate prefetch buffer would. Instead, while a tile is solved its
+//    successor is prefetched into L2, so that the next copies wait less.
 #include "dp_small.cuh"
 
 namespace dc {
@@ -54,7 +55,8 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
                        const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
                        int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,
                        int32_t *__restrict__ nseg, int32_t *__restrict__ status,
-                       uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list)
+                       uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list,
+                       bool pairs)
 {
     using K = Small<L, uint32_t, kKeepCols>;
     constexpr int W = (L - 1 + 31) / 32;
@@ -73,7 +75,14 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         const int64_t base = tile * 32;
         const int rows = rows_of(tile);
         __syncwarp();  // every lane is done with the table: stage the tile's rows there
-        stage_tile<L>(stC, stX, comp, xfer, base, rows, lane);
+        stage_tile<L>(stC, stX, comp, xfer, base, rows, lane, pairs);
+        if (tile + gridDim.x < tiles) {  // the warp's next tile into L2, one 128-byte line per lane and array
+            const int64_t nbase = (tile + gridDim.x) * 32;
+            if (lane * 16 < rows_of(tile + gridDim.x) * L) {
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(comp + nbase * L + lane * 16));
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(xfer + nbase * L + lane * 16));
+            }
+        }
         const int64_t i = base + lane;
         const bool active = lane < rows;
         const int64_t dti = active ? __ldg(dt + i) : 0;
@@ -174,7 +183,8 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;
     small_dense_kernel<L, FWD><<<unsigned(grid), 32, K32::kWarpBytes, stream>>>(
-        batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list);
+        batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list,
+        ((reinterpret_cast<uintptr_t>(comp) | reinterpret_cast<uintptr_t>(xfer)) & 15u) == 0);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     // the list length is known on the device only: persistent warps (4 per SM)

@@ -30,9 +30,15 @@ __host__ __device__ constexpr int cell2(int L, int m, int n)
     return (n - 2) * L - (n - 2) * (n - 1) / 2 + (m - n);
 }
 
-// Row stride of the staging buffer in int64 units: odd, so that the 16 lanes of a
-// half-warp reading 64-bit words of their own rows hit 16 distinct bank pairs.
-__host__ __device__ constexpr int stage_stride(int L) { return (L % 2 == 0) ? L + 1 : L; }
+// Row stride of the staging buffer in int64 units. Odd L: the odd stride L, so
+// that the 16 lanes of a half-warp reading 64-bit words of their own rows hit 16
+// distinct bank pairs. Even L: rows are copied and read as 16-byte pairs, so the
+// stride is even (16-byte aligned rows) and 2 mod 4, so that the 8 lanes of a
+// quarter-warp reading 16 bytes of their own rows hit 8 distinct 4-bank groups.
+__host__ __device__ constexpr int stage_stride(int L)
+{
+    return (L % 2 == 1) ? L : (L % 4 == 2 ? L : L + 2);
+}
 
 // Stored columns 2..C with C = min(keep, L-1); KEEP = L keeps them all.
 template <int L, typename T, int KEEP>
@@ -193,16 +199,17 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
 //   B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[m][1] = FC[L] + P[m],
 //   X[L][n] = B[L][n] + n*dt + P[L];
 // the next column's A[m] is that minimum less dt;
-// backward (BC = compute prefix, NGT[k] = -(transfer prefix)): with
-// E = X - n*dt - S[m],
-//   E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),  E[m][1] = BC[m],
-//   X[L][n] = E[L][n] + n*dt + S[L].
-// Both are min_k max(u[m] + V[k], C[k]) with a row constant u and the previous
-// column C in the max operand. Each candidate differs from Eq. 8/9's by a
+// backward (BC = compute prefix, NGT[k] = -(transfer prefix), U = BC - dt):
+// with F = X - dt - S[m],
+//   F[m][n] - dt = min_k max(U[m] + NGT[k], F[k][n-1]),  F[m][1] = BC[m],
+//   X[L][n] = F[L][n] + dt + S[L];
+// the next column's F[m] is that minimum plus dt.
+// Both are min_k max(U[m] + V[k], C[k]) with a row constant U, the same in every
+// column, and the previous column C in the max operand. Each candidate differs from Eq. 8/9's by a
 // constant of its row, so every argmin is the same. All values and sums lie in
 // [-2^31, 2^31) when the capped bound L*dt + sum(comp) + sum(capped xfer) is
 // below 2^31; other instances take the 64-bit pass. The table stores A (forward)
-// or E (backward) for columns 1..kKeepCols and the row U (U = Q forward, BC
+// or F (backward) for columns 1..kKeepCols and the row U (Q forward, BC - dt
 // backward); V (G forward, NGT backward) stays in registers.
 
 // Minimum of c[0..cnt-1] (cnt a compile-time constant after unrolling): two
@@ -231,31 +238,32 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
                                        int &best_s)
 {
     using K = Small<L, uint32_t, kKeepCols>;
-    // forward: U = Q, V = G, col = A; backward: U = BC, V = NGT, col = E
+    // forward: U = Q, V = G, col = A; backward: U = BC - dt, V = NGT, col = F
+    const int32_t dt2 = 2 * dt;
     int32_t col[L + 1];
 #pragma unroll
     for (int m = 1; m <= L; ++m) {
-        col[m] = FWD ? fcL + U[m] - dt : U[m];
+        col[m] = FWD ? fcL + U[m] - dt : U[m] + dt;
         if (m < L) lw[32 * (K::kOffC1 + m)] = col[m];  // for the traceback
     }
-    bestV = (FWD ? fcL : U[L]) + dt;
+    bestV = FWD ? fcL + dt : U[L] + dt2;
     best_s = 1;
 #pragma unroll
     for (int n = 2; n <= L; ++n) {
-        int32_t last = 0;  // B[L][n] or E[L][n]
+        int32_t last = 0;  // B[L][n] (forward) or F[L][n] - dt (backward)
 #pragma unroll
         for (int m = L; m >= n; --m) {  // descending: column n overwrites column n-1 in place
             const int cnt = m - n + 1;  // k = n-1 .. m-1
-            const int32_t u = FWD ? U[m] : U[m] - (n - 1) * dt;
+            const int32_t u = U[m];
             int32_t c[L];
 #pragma unroll
             for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(u, V[n - 1 + j], col[n - 1 + j]);
             const int32_t b = min_fold3<L>(c, cnt);
             if (m == L) last = FWD ? b - U[L] : b;
-            col[m] = FWD ? b - dt : b;
+            col[m] = FWD ? b - dt : b + dt;
             if (n <= K::kLast) lw[32 * cell2(L, m, n)] = col[m];
         }
-        const int32_t v = last + n * dt;
+        const int32_t v = FWD ? last + n * dt : last + dt2;  // X[L][n] - P[L] or X[L][n] - S[L]
         if (v < bestV) {  // strict: the lowest n wins ties
             bestV = v;
             best_s = n;
@@ -265,7 +273,7 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
 
 // The fill, the traceback and the outputs of one instance in shifted form, from
 // its U and V rows (forward: U = dt + capped transfer prefix, V = FC[L] - compute
-// prefix; backward: U = compute prefix, V = -capped transfer prefix) and the raw
+// prefix; backward: U = compute prefix - dt, V = -capped transfer prefix) and the raw
 // transfer sum. Returns false (writing nothing) when the traceback needs a column
 // the pass did not keep.
 template <int L, bool FWD>
@@ -292,11 +300,10 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
     uint32_t word = 0;
     int err = 0;
     int m = L, n = s;
-    int32_t target = bestV - s * dt + (FWD ? U[L] : 0);  // B[L][s] + Q[L] or E[L][s]
+    int32_t target = FWD ? bestV - s * dt + U[L] : bestV - 2 * dt;  // B[L][s] + Q[L] or F[L][s] - dt
     while (n > 1) {
         const int nm1 = n - 1;
-        const int32_t um = lds(lw, K::kOffR + m);
-        const int32_t u = FWD ? um : um - nm1 * dt;
+        const int32_t u = lds(lw, K::kOffR + m);
         // cell (k, n-1) is base + k; column 1 has its own row of the table
         const int base = nm1 == 1 ? K::kOffC1 : cell2(L, 0, nm1);
         uint32_t hit = 0u;
@@ -312,8 +319,8 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
         }
         const int k = __ffs(int(hit)) - 1;
         word |= 1u << ((k - 1) & 31);
-        const int32_t fk = lds(lw, base + k);  // the cell (k, n-1): B + Q[k] = A + dt, or E
-        target = FWD ? fk + dt : fk;
+        const int32_t fk = lds(lw, base + k);  // the cell (k, n-1): B + Q[k] = A + dt, or F - dt
+        target = FWD ? fk + dt : fk - dt;
         m = k;
         n = nm1;
     }
@@ -333,7 +340,7 @@ __device__ __forceinline__ void shifted_uv(const uint64_t (&Pc)[L + 1], const ui
     const int32_t fcL = int32_t(Pc[L]);
 #pragma unroll
     for (int m = 0; m <= L; ++m) {
-        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]);
+        U[m] = FWD ? dt + int32_t(Px[m]) : int32_t(Pc[m]) - dt;
         V[m] = FWD ? fcL - int32_t(Pc[m]) : -int32_t(Px[m]);
     }
 }
@@ -356,19 +363,36 @@ __device__ __forceinline__ bool fast_uv(const int64_t *rc, const int64_t *rx, in
     constexpr int kCompBits = 31 - ceil_log2(L);
     uint32_t cl[L], xl[L];
     uint32_t hor = uint32_t(uint64_t(dti) >> 31), cor = 0u, tc = 0u;
+    if constexpr (L % 2 == 0) {  // 16-byte rows: two costs per load
 #pragma unroll
-    for (int r = 0; r < L; ++r) {
-        const int col = FWD ? r : L - 1 - r;
-        const uint2 c = *reinterpret_cast<const uint2 *>(rc + col);
-        const uint2 x = *reinterpret_cast<const uint2 *>(rx + col);
-        cl[r] = c.x;
-        xl[r] = x.x;
-        hor |= c.y | x.y;
-        cor |= c.x;
-        tc += c.x;
+        for (int q = 0; q < L; q += 2) {
+            const uint4 c = *reinterpret_cast<const uint4 *>(rc + q);
+            const uint4 x = *reinterpret_cast<const uint4 *>(rx + q);
+            const int r0 = FWD ? q : L - 1 - q, r1 = FWD ? q + 1 : L - 2 - q;
+            cl[r0] = c.x;
+            cl[r1] = c.z;
+            xl[r0] = x.x;
+            xl[r1] = x.z;
+            hor |= c.y | x.y;
+            hor |= c.w | x.w;
+            cor |= c.x | c.z;
+            tc += c.x + c.z;
+        }
+    } else {
+#pragma unroll
+        for (int r = 0; r < L; ++r) {
+            const int col = FWD ? r : L - 1 - r;
+            const uint2 c = *reinterpret_cast<const uint2 *>(rc + col);
+            const uint2 x = *reinterpret_cast<const uint2 *>(rx + col);
+            cl[r] = c.x;
+            xl[r] = x.x;
+            hor |= c.y | x.y;
+            cor |= c.x;
+            tc += c.x;
+        }
     }
     if ((hor | (cor >> kCompBits)) != 0u) return false;
-    uint32_t u = FWD ? uint32_t(dti) : 0u, v = FWD ? tc : 0u;
+    uint32_t u = FWD ? uint32_t(dti) : 0u - uint32_t(dti), v = FWD ? tc : 0u;
     U[0] = int32_t(u);
     V[0] = int32_t(v);
     uint64_t px = 0, xr = 0;
@@ -397,22 +421,41 @@ __device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src)
     const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
     asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(gmem_src) : "memory");
 }
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src)
+{
+    const uint32_t d = uint32_t(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// Issue the copies of tile `base` (rows base..base+rows-1) into the staging area.
+// Issue the copies of tile `base` (rows base..base+rows-1) into the staging area:
+// 16-byte copies of cost pairs when L is even and both cost arrays are 16-byte
+// aligned (`pairs`; every pair then starts on a 16-byte boundary on both sides),
+// else 8-byte copies.
 template <int L>
 __device__ __forceinline__ void stage_tile(int64_t *stC, int64_t *stX, const int64_t *comp,
-                                           const int64_t *xfer, int64_t base, int rows, int lane)
+                                           const int64_t *xfer, int64_t base, int rows, int lane,
+                                           bool pairs)
 {
     constexpr int kStride = stage_stride(L);
     const int64_t *gC = comp + base * L;
     const int64_t *gX = xfer + base * L;
-    const int nel = rows * L;
-    for (int e = lane; e < nel; e += 32) {
-        const int r = e / L, cidx = e - r * L;
-        cp_async8(stC + r * kStride + cidx, gC + e);
-        cp_async8(stX + r * kStride + cidx, gX + e);
+    if (L % 2 == 0 && pairs) {
+        constexpr int H = L / 2 > 0 ? L / 2 : 1;  // pairs per row
+        const int np = rows * H;
+        for (int p = lane; p < np; p += 32) {
+            const int r = p / H, cidx = 2 * (p - r * H);
+            cp_async16(stC + r * kStride + cidx, gC + 2 * p);
+            cp_async16(stX + r * kStride + cidx, gX + 2 * p);
+        }
+    } else {
+        const int nel = rows * L;
+        for (int e = lane; e < nel; e += 32) {
+            const int r = e / L, cidx = e - r * L;
+            cp_async8(stC + r * kStride + cidx, gC + e);
+            cp_async8(stX + r * kStride + cidx, gX + e);
+        }
     }
     cp_async_commit();
 }

@@ -122,6 +122,33 @@ def test_dp_wide_latency_small_compute_parity(dc, L):
         _check_direction(dc, d, comp, xfer, dt, f"wide-latency L={L} dir={d}")
 
 
+@pytest.mark.parametrize("L", [2, 6, 8, 13, 14, 16])
+@pytest.mark.parametrize("which", ["both", "xfer"])
+def test_dp_unaligned_cost_arrays(dc, L, which):
+    """Cost arrays starting 8 bytes past a 16-byte boundary: the short-L pass then
+    stages single costs instead of 16-byte pairs. Same outputs as the oracle."""
+    import torch
+    B = 1000 + 17
+    comp, xfer, dt = wl.random_instances(900 + L, B, L, 0, 100_000, 0, 10_000)
+
+    def shifted(a):
+        buf = torch.empty(a.size + 1, dtype=torch.int64, device="cuda")
+        v = buf[1:].view(a.shape)
+        v.copy_(torch.from_numpy(np.ascontiguousarray(a)))
+        assert v.data_ptr() % 16 == 8
+        return v
+
+    W = dc.words(L)
+    for d in (FWD, BWD):
+        c = shifted(comp) if which == "both" else _dev(comp)
+        out = dc.schedule(d, c, shifted(xfer), _dev(dt))
+        torch.cuda.synchronize()
+        got = {k: v.cpu().numpy() for k, v in out.items()}
+        got["bits"] = got["bits"].view(np.uint32)[:, :W] if W else np.zeros((B, 0), np.uint32)
+        exp = oracle.schedule_batch(d, comp, xfer, dt, nthreads=NTHREADS)
+        _assert_same(got, exp, f"unaligned {which} L={L} dir={d}")
+
+
 @pytest.mark.parametrize("L", [8, 16, 54, 100])
 def test_dp_status_faults_per_instance(dc, L):
     B = 300
