@@ -147,6 +147,9 @@ def test_dp_unaligned_cost_arrays(dc, L, which):
         got["bits"] = got["bits"].view(np.uint32)[:, :W] if W else np.zeros((B, 0), np.uint32)
         exp = oracle.schedule_batch(d, comp, xfer, dt, nthreads=NTHREADS)
         _assert_same(got, exp, f"unaligned {which} L={L} dir={d}")
+        # the replay of those decisions from the same unaligned arrays
+        rep = dc.eval_timeline(d, c, shifted(xfer), _dev(dt), out["bits"][:, :max(W, 1)].contiguous())
+        assert np.array_equal(rep.cpu().numpy(), exp["makespan"]), f"replay unaligned {which} L={L}"
 
 
 @pytest.mark.parametrize("L", [8, 16, 54, 100])
