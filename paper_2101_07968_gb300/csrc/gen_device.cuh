@@ -57,6 +57,17 @@ __device__ __forceinline__ int64_t loguniform(const Tab &knots, uint64_t r)
 // precomputed once per divisor: q = mulhi(a, m) is floor(a/d) or one less,
 // because a*m/2^64 >= a/d - a*(1 + ((2^64-1) mod d))/(d*2^64) > a/d - 1/4; one
 // remainder step makes it exact.
+__device__ __forceinline__ void floor_div(uint64_t a, uint64_t d, uint64_t m, uint64_t &q,
+                                          uint64_t &r)
+{
+    q = __umul64hi(a, m);
+    r = a - q * d;
+    if (r >= d) {
+        ++q;
+        r -= d;
+    }
+}
+
 __device__ __forceinline__ uint64_t ceil_div(uint64_t a, uint64_t d, uint64_t m)
 {
     uint64_t q = __umul64hi(a, m);
@@ -131,8 +142,18 @@ __device__ __forceinline__ void layer_costs(const GenParams &g, const InstanceDr
                                             int64_t &bc, int64_t &xfer)
 {
     xfer = int64_t(ceil_div(uint64_t(g.bits) * 1000u * uint64_t(params), d.bw, d.mbw));
-    fc = int64_t(ceil_div(uint64_t(flops), d.rate, d.mrate));
-    bc = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), d.rate, d.mrate));
+    if (g.bwd_mult == 2) {
+        // flops = q*rate + r (0 <= r < rate): ceil(flops/rate) = q + (r > 0) and
+        // ceil(2*flops/rate) = 2q + ceil(2r/rate) = 2q + (r > 0) + (2r > rate)
+        uint64_t q, r;
+        floor_div(uint64_t(flops), d.rate, d.mrate, q, r);
+        const uint64_t up = r != 0 ? 1u : 0u;
+        fc = int64_t(q + up);
+        bc = int64_t(2 * q + up + (2 * r > d.rate ? 1u : 0u));
+    } else {
+        fc = int64_t(ceil_div(uint64_t(flops), d.rate, d.mrate));
+        bc = int64_t(ceil_div(uint64_t(g.bwd_mult) * uint64_t(flops), d.rate, d.mrate));
+    }
 }
 
 }  // namespace dc
