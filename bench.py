@@ -127,13 +127,13 @@ def load_json(path):
 
 
 def dp_source_hash() -> str:
-    """Hash of the DP sources' code (comments and blank space removed), which a
-    traffic record must match to be reported."""
+    """Hash of the code (comments and blank space removed) of the sources the
+    short-L dense pass is built from, which a traffic record must match to be
+    reported."""
     import hashlib
     import re
     h = hashlib.sha256()
-    for name in ("dp_small.cu", "dp_small.cuh", "dp_mid.cu", "dp_group.cu", "common.cuh",
-                 "dynacomm_abi.cu"):
+    for name in ("dp_small.cu", "dp_small.cuh", "gen_device.cuh", "common.cuh"):
         with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name)) as f:
             code = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
         code = re.sub(r"//[^\n]*", "", code)
