@@ -53,7 +53,7 @@ namespace {
 
 constexpr int kB = 8;  // rows per register block
 constexpr int kKeep = 8;  // last column kept for the traceback
-constexpr int kMidSplitL = 41;  // from this L on, two warps share a forward tile
+constexpr int kMidSplitL = 41;  // from this L on, two warps share a tile
 
 __host__ __device__ inline int mid_keep_last(int L) { return L - 1 < kKeep ? L - 1 : kKeep; }
 // stored cell (m, n), 2 <= n <= keep_last
@@ -347,13 +347,13 @@ __global__ void __launch_bounds__(32 * NW)
         int32_t target = FWD ? bestV - s * dt32 + U[32 * L] : bestV - 2 * dt32;  // B[L][s] + Q[L] or F[L][s] - dt
         while (n > 1) {
             const int32_t uu = U[32 * m];
-            // candidates in groups of 4 (loads issued together, lowest match wins)
+            // candidates in groups of 8 (loads issued together, lowest match wins)
             int k = -1;
             int32_t fk = 0;
-            for (int k0 = n - 1; k0 < m && k < 0; k0 += 4) {
-                int32_t f[4], v[4];
+            for (int k0 = n - 1; k0 < m && k < 0; k0 += 8) {
+                int32_t f[8], v[8];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
+                for (int u = 0; u < 8; ++u) {
                     const int kk = k0 + u < m ? k0 + u : m - 1;  // stay inside column n-1
                     v[u] = pv[32 * kk].y;
                     if (n - 1 == 1)  // column 1 from U
@@ -362,7 +362,7 @@ __global__ void __launch_bounds__(32 * NW)
                         f[u] = int32_t(myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots]);
                 }
 #pragma unroll
-                for (int u = 3; u >= 0; --u) {
+                for (int u = 8 - 1; u >= 0; --u) {
                     if (k0 + u < m && __viaddmax_s32(uu, v[u], f[u]) == target) {
                         k = k0 + u;
                         fk = f[u];
@@ -422,17 +422,17 @@ cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
                        uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream)
 {
-    // two warps per tile once the lane slices limit the resident warps: measured
-    // faster for the forward pass from L = 41 on; the backward pass measured no
-    // gain (its warp 1 waits out longer tracebacks), so it keeps one warp
-    if (forward)
-        return L >= kMidSplitL
-                   ? launch_mid_nw<true, 2>(batch, L, comp, xfer, dt, makespan, bits, nseg,
+    // two warps per tile once the lane slices limit the resident warps (measured
+    // faster from L = 41 on)
+    if (L >= kMidSplitL)
+        return forward ? launch_mid_nw<true, 2>(batch, L, comp, xfer, dt, makespan, bits, nseg,
+                                                status, ticket, list_count, list, tb, stream)
+                       : launch_mid_nw<false, 2>(batch, L, comp, xfer, dt, makespan, bits, nseg,
+                                                 status, ticket, list_count, list, tb, stream);
+    return forward ? launch_mid_nw<true, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg,
                                             status, ticket, list_count, list, tb, stream)
-                   : launch_mid_nw<true, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg,
-                                            status, ticket, list_count, list, tb, stream);
-    return launch_mid_nw<false, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                                   ticket, list_count, list, tb, stream);
+                   : launch_mid_nw<false, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg,
+                                             status, ticket, list_count, list, tb, stream);
 }
 
 }  // namespace dc
