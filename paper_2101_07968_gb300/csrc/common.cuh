@@ -11,9 +11,9 @@
 namespace dc {
 
 constexpr int kSmallLMax = 16;       // unrolled thread-per-instance kernel: 1 <= L <= 16
-constexpr int kMidLMax = 64;         // looped thread-per-instance kernel: 17 <= L <= 64
+constexpr int kMidLMax = 256;        // looped thread-per-instance kernel: 17 <= L <= 256
 constexpr int kSmemTableLMax = 64;   // group kernel keeps its DP table on chip up to here
-constexpr int64_t kMidSlots = 152 * 16 * 32;  // traceback slots of the looped kernel
+constexpr int64_t kMidSlots = 152 * 16 * 32;  // traceback slots of the looped kernel (L <= 64)
 constexpr int64_t kRangeLimit = int64_t(1) << 52;
 constexpr uint64_t kNarrowLimit = 0xFFFFFFFEull;  // bound that lets a DP run in 32 bits
 // capped bound under which the shifted form of a DP runs in signed 32 bits
@@ -41,12 +41,14 @@ inline int64_t table_slots(int L)
     return s;
 }
 
-size_t mid_scratch_bytes(int L);  // dp_mid.cu
+size_t mid_scratch_bytes(int64_t batch, int L);  // dp_mid.cu
 
 struct Workspace {
     // Layout: [0, 256) header (work-list counter, tile ticket), [256, 256 + 4*batch)
     // work list (L <= kMidLMax), then, 256-aligned, the looped kernel's traceback
-    // slots (17 <= L <= 64) or the per-CTA DP tables of the group kernel (L > 64).
+    // slots (17 <= L <= kMidLMax), then, 256-aligned, the per-CTA DP tables of the
+    // group kernel (L > kSmemTableLMax: the looped kernel's work list or, above
+    // kMidLMax, the whole batch).
     static size_t list_bytes(int64_t batch, int L)
     {
         return L <= kMidLMax ? size_t(batch) * 4 : 0;
@@ -61,10 +63,15 @@ struct Workspace {
         int64_t s = table_slots(L);
         return size_t(batch < s ? batch : s);
     }
+    static size_t group_tables_offset(int64_t batch, int L)
+    {
+        if (L > kSmallLMax && L <= kMidLMax)
+            return (table_offset(batch, L) + mid_scratch_bytes(batch, L) + 255) / 256 * 256;
+        return table_offset(batch, L);
+    }
     static size_t bytes(int64_t batch, int L)
     {
-        if (L > kSmallLMax && L <= kMidLMax) return table_offset(batch, L) + mid_scratch_bytes(L);
-        return table_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
+        return group_tables_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
     }
 };
 

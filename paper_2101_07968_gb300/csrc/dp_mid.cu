@@ -1,4 +1,4 @@
-// Thread-per-instance DynaComm DP for 17 <= L <= 64 (Eq. 8 / Algorithm 3 and
+// Thread-per-instance DynaComm DP for 17 <= L <= 256 (Eq. 8 / Algorithm 3 and
 // Eq. 9 / Algorithm 4), 32-bit arithmetic, runtime loops.
 //
 // Same processing-order template as the other kernels:
@@ -40,22 +40,32 @@
 //    put on a work list that the CTA-per-instance kernel solves afterwards;
 //  * persistent CTAs claim 32-instance tiles from an atomic ticket, so the
 //    long, uneven per-tile work balances across the GPU. The lane slices take
-//    3*(L+1) words per lane and limit the resident warps, so for long rows two
-//    warps share a tile (same slices, half the shared memory per warp): the
-//    column's row blocks are dealt to them in a snake (0, 3, 4, 7 / 1, 2, 5, 6),
-//    each warp keeps its results in registers until both have read column n-1
-//    (a CTA barrier), then both write column n and meet at a second barrier.
-//    Warp 0 reads the rows and does the traceback.
+//    3*(L+1) words per lane and limit the resident warps, so for long rows 2, 4
+//    or 8 warps share a tile (same slices, less shared memory per warp): the
+//    column's row blocks are dealt to them in a snake, each warp keeps its
+//    results in registers until all have read column n-1 (a CTA barrier), then
+//    all write column n and meet at a second barrier. Warp 0 reads the rows and
+//    does the traceback.
 #include "common.cuh"
 
 namespace dc {
 namespace {
 
 constexpr int kB = 8;  // rows per register block
-constexpr int kKeep = 8;  // last column kept for the traceback
-constexpr int kMidSplitL = 41;  // from this L on, two warps share a tile
+constexpr int kQ = 4;  // row blocks of a column per warp, at most (L <= 32 * warps)
 
-__host__ __device__ inline int mid_keep_last(int L) { return L - 1 < kKeep ? L - 1 : kKeep; }
+// warps sharing a tile: the lane slices take 3*(L+1) words per lane and limit
+// the resident warps, so longer rows spread a tile over more warps (measured
+// faster from L = 41 on)
+__host__ __device__ inline int mid_warps(int L) { return L <= 40 ? 1 : L <= 64 ? 2 : L <= 128 ? 4 : 8; }
+
+// last column kept for the traceback (a traceback of s segments reads columns
+// 1..s-1): 8 up to L = 64, 16 beyond (deeper optima are more common there)
+__host__ __device__ inline int mid_keep_last(int L)
+{
+    const int keep = L <= 64 ? 8 : 16;
+    return L - 1 < keep ? L - 1 : keep;
+}
 // stored cell (m, n), 2 <= n <= keep_last
 __host__ __device__ inline int mid_cell(int L, int m, int n)
 {
@@ -65,6 +75,15 @@ __host__ __device__ inline int mid_cells(int L)
 {
     const int c = mid_keep_last(L);
     return c >= 2 ? mid_cell(L, L, c) + 1 : 0;
+}
+// traceback slots (one per lane of a launched CTA): about one resident wave of
+// CTAs (kMidSlots up to L = 64), and no more than the batch's tiles need
+__host__ __device__ inline int64_t mid_slots(int64_t batch, int L)
+{
+    const int nw = mid_warps(L);
+    const int64_t wave = nw <= 2 ? kMidSlots : int64_t(152) * 32 * (nw == 4 ? 4 : 2);
+    const int64_t need = (batch + 31) / 32 * 32;
+    return need < wave ? need : wave;
 }
 
 // Rows -> the lane slices: U (Q forward, BC - dt backward) at 32*v, and the
@@ -228,8 +247,9 @@ __device__ __forceinline__ void mid_rows(int L, int n, int b, int &top, int &bot
 }
 
 // Block of warp w for its q-th slot when NW warps share a column: a snake over
-// the blocks (0, 3, 4, 7 to warp 0 and 1, 2, 5, 6 to warp 1 for NW = 2), which
-// evens out the work of the upper (longer) and lower blocks.
+// the blocks (0, 3, 4, 7 to warp 0 and 1, 2, 5, 6 to warp 1 for NW = 2; rows
+// 0..NW-1 left to right, the next NW right to left, and so on), which evens out
+// the work of the upper (longer) and lower blocks.
 template <int NW>
 __device__ __forceinline__ int mid_block_of(int q, int w)
 {
@@ -259,7 +279,6 @@ __global__ void __launch_bounds__(32 * NW)
     uint32_t *myslot = tb + slot;  // cell c at myslot[c * nslots]
     const int keep = mid_keep_last(L);
     const int64_t tiles = (batch + 31) / 32;
-    constexpr int kQ = (kMidLMax / kB + NW - 1) / NW;  // blocks per warp and column, at most
 
     for (;;) {
         if (threadIdx.x == 0) s_tile = atomicAdd(ticket, 1u);
@@ -342,7 +361,9 @@ __global__ void __launch_bounds__(32 * NW)
         }
 
         // ---- traceback: lowest k whose candidate equals the cell
-        uint32_t word0 = 0u, word1 = 0u;  // L <= 64: W <= 2
+        // decision words 0 and 1 in registers; words 2.. (L > 65) set in place
+        uint32_t word0 = 0u, word1 = 0u;
+        for (int w = 2; w < W; ++w) bits[i * W + w] = 0u;
         int err = 0, m = L, n = s;
         int32_t target = FWD ? bestV - s * dt32 + U[32 * L] : bestV - 2 * dt32;  // B[L][s] + Q[L] or F[L][s] - dt
         while (n > 1) {
@@ -375,8 +396,10 @@ __global__ void __launch_bounds__(32 * NW)
             }
             if (k - 1 < 32)
                 word0 |= 1u << (k - 1);
-            else
+            else if (k - 1 < 64)
                 word1 |= 1u << (k - 33);
+            else
+                bits[i * W + ((k - 1) >> 5)] |= 1u << ((k - 1) & 31);
             target = FWD ? fk + dt32 : fk - dt32;  // the cell (k, n-1): B + Q[k] = A + dt, or F - dt
             m = k;
             n -= 1;
@@ -404,35 +427,38 @@ cudaError_t launch_mid_nw(int64_t batch, int L, const int64_t *comp, const int64
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    int64_t grid = kMidSlots / 32;
-    const int64_t tiles = (batch + 31) / 32;
-    if (grid > tiles) grid = tiles;
+    const int64_t slots = mid_slots(batch, L);
+    const int64_t grid = slots / 32;
     mid_kernel<FWD, NW><<<unsigned(grid), 32 * NW, smem, stream>>>(
         batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket, list_count, list, tb,
-        kMidSlots);
+        slots);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-size_t mid_scratch_bytes(int L) { return size_t(kMidSlots) * size_t(mid_cells(L)) * 4; }
+size_t mid_scratch_bytes(int64_t batch, int L)
+{
+    return size_t(mid_slots(batch, L)) * size_t(mid_cells(L)) * 4;
+}
 
 cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
                        uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream)
 {
-    // two warps per tile once the lane slices limit the resident warps (measured
-    // faster from L = 41 on)
-    if (L >= kMidSplitL)
-        return forward ? launch_mid_nw<true, 2>(batch, L, comp, xfer, dt, makespan, bits, nseg,
-                                                status, ticket, list_count, list, tb, stream)
-                       : launch_mid_nw<false, 2>(batch, L, comp, xfer, dt, makespan, bits, nseg,
-                                                 status, ticket, list_count, list, tb, stream);
-    return forward ? launch_mid_nw<true, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg,
-                                            status, ticket, list_count, list, tb, stream)
-                   : launch_mid_nw<false, 1>(batch, L, comp, xfer, dt, makespan, bits, nseg,
-                                             status, ticket, list_count, list, tb, stream);
+#define DC_MID_LAUNCH(NW)                                                                        \
+    return forward ? launch_mid_nw<true, NW>(batch, L, comp, xfer, dt, makespan, bits, nseg,    \
+                                             status, ticket, list_count, list, tb, stream)       \
+                   : launch_mid_nw<false, NW>(batch, L, comp, xfer, dt, makespan, bits, nseg,   \
+                                              status, ticket, list_count, list, tb, stream);
+    switch (mid_warps(L)) {
+        case 1: DC_MID_LAUNCH(1)
+        case 2: DC_MID_LAUNCH(2)
+        case 4: DC_MID_LAUNCH(4)
+        default: DC_MID_LAUNCH(8)
+    }
+#undef DC_MID_LAUNCH
 }
 
 }  // namespace dc

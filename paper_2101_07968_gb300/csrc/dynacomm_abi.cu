@@ -37,13 +37,18 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
         e = launch_mid(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket,
                        count, list, tb, stream);
         if (e != cudaSuccess) return e;
-        const int64_t grid = batch < 152 * 8 ? batch : 152 * 8;
+        if (L <= kSmemTableLMax) {  // tables of the listed instances in shared memory
+            const int64_t grid = batch < 152 * 8 ? batch : 152 * 8;
+            return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
+                                count, list, nullptr, grid, stream);
+        }
         return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                            count, list, nullptr, grid, stream);
+                            count, list, ws + Workspace::group_tables_offset(batch, L),
+                            int64_t(Workspace::slots(batch, L)), stream);
     }
     const int64_t slots = int64_t(Workspace::slots(batch, L));
     return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                        nullptr, nullptr, ws + Workspace::table_offset(batch, L), slots,
+                        nullptr, nullptr, ws + Workspace::group_tables_offset(batch, L), slots,
                         stream);
 }
 

@@ -47,10 +47,16 @@ def test_workspace_query(lib):
     assert dc.dc_schedule_workspace_bytes(10, 0) == 0
     assert dc.dc_schedule_workspace_bytes(10, 4097) == 0
     assert dc.dc_schedule_workspace_bytes(1000, 16) >= 256 + 4000
-    # 17 <= L <= 64: work list plus fixed per-thread traceback slots
+    # 17 <= L <= 256: work list plus per-thread traceback slots, one per lane of
+    # the launched CTAs: as many as the batch's tiles need, up to about one
+    # resident wave (then fixed, so only the work list grows)
     mid = dc.dc_schedule_workspace_bytes(1000, 54)
     assert mid >= 256 + 4000 and mid == dc.dc_schedule_workspace_bytes(1000, 54)
-    assert abs(dc.dc_schedule_workspace_bytes(2000, 54) - mid - 4000) < 256
+    assert dc.dc_schedule_workspace_bytes(2000, 54) > mid + 4000
+    big = dc.dc_schedule_workspace_bytes(200_000, 54)
+    assert abs(dc.dc_schedule_workspace_bytes(300_000, 54) - big - 400_000) < 256
+    # above L = 64 the listed instances also get DP-table slots
+    assert dc.dc_schedule_workspace_bytes(1000, 65) > dc.dc_schedule_workspace_bytes(1000, 64)
     # long L: one DP-table slot per concurrently solved instance
     one = dc.dc_schedule_workspace_bytes(1, 1024)
     assert one >= 1024 * 1025 // 2 * 8

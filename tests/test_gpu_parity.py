@@ -64,7 +64,7 @@ def _check_direction(dc, direction, comp, xfer, dt, label=""):
 
 
 # ------------------------------------------------------------------ DP parity
-SMALL_LS = list(range(1, 21)) + [31, 32, 33, 40, 41, 48, 54, 63, 64, 65, 96, 130]
+SMALL_LS = list(range(1, 21)) + [31, 32, 33, 40, 41, 48, 54, 63, 64, 65, 96, 128, 129, 130, 256]
 
 
 @pytest.mark.parametrize("L", SMALL_LS)
