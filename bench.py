@@ -596,9 +596,9 @@ def run_ours(args):
     hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
     dp_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
     # kernels of this library per step: the generator; per direction the 32-bit
-    # pass and the pass over its work list (L <= 64) or the per-instance kernel
-    # alone (L > 64); the two timeline replays
-    launches_per_step = 1 + 2 * (2 if L <= 64 else 1) + 2
+    # pass and the pass over its work list (L <= 256) or the per-instance kernel
+    # alone (L > 256); the two timeline replays
+    launches_per_step = 1 + 2 * (2 if L <= 256 else 1) + 2
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,

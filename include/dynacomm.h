@@ -111,7 +111,8 @@ dc_status dc_profile_gen(const dc_profile_cfg *cfg, int64_t *fc, int64_t *pt, in
 
 /* ------------------------------------------------------------------------
  * dc_schedule_workspace_bytes -- device scratch a schedule call needs for
- * (batch, L): a work list for instances whose values need 64-bit arithmetic,
+ * (batch, L): a work list for instances whose values need 64-bit arithmetic
+ * (L <= 256), traceback slots of the thread-per-instance kernel (17 <= L <= 256)
  * and, for L > 64, per-CTA DP tables. Pure host function, no CUDA call.
  * ---------------------------------------------------------------------- */
 size_t dc_schedule_workspace_bytes(int64_t batch, int32_t L);
