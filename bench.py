@@ -599,6 +599,24 @@ def run_ours(args):
     # pass and the pass over its work list (L <= 256) or the per-instance kernel
     # alone (L > 256); the two timeline replays
     launches_per_step = 1 + 2 * (2 if L <= 256 else 1) + 2
+    # both roofs of the DP pass; the one it comes closer to (the larger minimal
+    # time at peak) binds and is reported, the other rides along
+    alu_roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "Gtransitions/s",
+                "frac": achieved / peak,
+                "peak_source": f"{sms} SMs x 64 integer-ALU lanes x {MAX_SM_MHZ} MHz / "
+                               f"{ALU_OPS_PER_TRANSITION} ALU instructions per transition",
+                "peak_probe": roof[0] / 1e9,
+                "peak_probe_source": "register-only loop of the 32-bit passes' op mix, "
+                                     "all SMs, measured in this run",
+                "peak_u64_probe": roof[1] / 1e9}
+    hbm_roof = {"bound": "hbm", "achieved": dp_gbs, "peak": hbm_peak, "unit": "GB/s",
+                "frac": dp_gbs / hbm_peak,
+                "bytes_per_instance_direction": dp_bytes(L),
+                "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}
+    binding, other = ((alu_roof, hbm_roof) if alu_roof["frac"] >= hbm_roof["frac"]
+                      else (hbm_roof, alu_roof))
+    roofline = dict(binding, kernel="dp_schedule (forward + backward)", traffic=traffic,
+                    other_roof=other)
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -613,18 +631,7 @@ def run_ours(args):
         "dp_transitions_per_s": trans * world / (ms * 1e-3),
         "breakdown_ms": {"profile_gen": gen_ms, "dp_forward": fwd_ms, "dp_backward": bwd_ms,
                          "eval_timeline_fwd_bwd": eval_ms},
-        "roofline": {"bound": "alu", "kernel": "dp_schedule (forward + backward)",
-                     "achieved": achieved, "peak": peak, "unit": "Gtransitions/s",
-                     "frac": achieved / peak, "traffic": traffic,
-                     "peak_source": f"{sms} SMs x 64 integer-ALU lanes x {MAX_SM_MHZ} MHz / "
-                                    f"{ALU_OPS_PER_TRANSITION} ALU instructions per transition",
-                     "peak_probe": roof[0] / 1e9,
-                     "peak_probe_source": "register-only loop of the 32-bit passes' op mix, "
-                                          "all SMs, measured in this run",
-                     "peak_u64_probe": roof[1] / 1e9,
-                     "hbm": {"achieved_gbs": dp_gbs, "peak_gbs": hbm_peak,
-                             "frac": dp_gbs / hbm_peak,
-                             "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}},
+        "roofline": roofline,
         "e2e": e2e,
         "cpu_baseline": cpu,
         "gpu_launches": launches_per_step * args.steps,
