@@ -40,3 +40,26 @@ def test_host_pipeline_matches_oracle(dc, name, batch, chunks):
             assert np.array_equal(host_out[(d, "bits")].numpy().view(np.uint32)[:, :W],
                                   exp["bits"])
             assert np.array_equal(host_out[(d, "replay")].numpy(), exp["makespan"])
+
+
+def test_host_pipeline_shared_transfer_buffer(dc):
+    """gt passed as the pt host buffer (equal transfer costs): copied once, the
+    same results as separate buffers."""
+    import torch
+    cfg = wl.with_batch(wl.config("vgg16"), 20_011)
+    ref = oracle.profile_gen(cfg)
+    assert np.array_equal(ref["pt"], ref["gt"])
+    sep = {k: torch.from_numpy(v).pin_memory() for k, v in ref.items()}
+    shared = dict(sep)
+    shared["gt"] = shared["pt"]
+    pipe = dc.HostPipeline(cfg["batch"], cfg["L"], chunks=5)
+    out_sep, out_shared = pipe.host_buffers(), pipe.host_buffers()
+    pipe.run(sep, out_sep)
+    torch.cuda.synchronize()
+    pipe.run(shared, out_shared)
+    torch.cuda.synchronize()
+    for k in out_sep:
+        assert torch.equal(out_sep[k], out_shared[k]), k
+    h_sep, _ = pipe.bytes_per_run(sep)
+    h_shared, _ = pipe.bytes_per_run(shared)
+    assert h_sep - h_shared == ref["gt"].nbytes
