@@ -11,7 +11,7 @@
 //             push (Eq. 2, 7): link_j = max(link_{j-1}, done_j) + dt + sum gt.
 // Inputs are checked like the solver's (negative -> -3, bound >= 2^52 -> -4).
 //
-// For L <= 32 a warp first copies its 32 instances' rows into shared memory with
+// For L <= 64 a warp first copies its 32 instances' rows into shared memory with
 // coalesced asynchronous copies (16-byte copies of cost pairs for even L; a row
 // stride at which every lane reads its own row without bank conflicts), then
 // replays its lane's row. Warps are persistent (one resident wave) and prefetch
@@ -26,7 +26,7 @@ int sm_count();  // SMs of the current device (dp_small.cu)
 
 namespace {
 
-constexpr int kStagedLMax = 32;
+constexpr int kStagedLMax = 64;
 constexpr int kEvalWarps = 4;
 
 struct Replay {
@@ -163,7 +163,11 @@ __global__ void __launch_bounds__(32 * kEvalWarps)
         const bool active = lane < rows;
         const int64_t i = base + lane;
         const int64_t d = active ? __ldg(dt + i) : 0;
-        const uint32_t word = (active && L > 1) ? __ldg(bits + i) : 0u;  // W = 1 for 2 <= L <= 32
+        const int W = words_for(L);  // 1 or 2 for L <= 64
+        const uint32_t w0 = (active && W > 0) ? __ldg(bits + i * W) : 0u;
+        const uint32_t w1 = (active && W > 1) ? __ldg(bits + i * W + 1) : 0u;
+        // break after processing position b + 1 (0-based b)
+        auto brk = [&](int b) { return ((b < 32 ? w0 >> b : w1 >> (b - 32)) & 1u) != 0u; };
         asm volatile("cp.async.wait_group 0;\n" ::: "memory");
         __syncwarp();
         if (!active) continue;
@@ -175,8 +179,8 @@ __global__ void __launch_bounds__(32 * kEvalWarps)
                 const longlong2 c = *reinterpret_cast<const longlong2 *>(rc + col);
                 const longlong2 x = *reinterpret_cast<const longlong2 *>(rx + col);
                 const int r = q + 1;
-                const bool cut0 = (word >> (r - 1)) & 1u;
-                const bool cut1 = (r + 1 == L) || ((word >> r) & 1u);
+                const bool cut0 = brk(r - 1);
+                const bool cut1 = (r + 1 == L) || brk(r);
                 if (FWD) {
                     rp.step<FWD>(c.x, x.x, uint64_t(d), cut0);
                     rp.step<FWD>(c.y, x.y, uint64_t(d), cut1);
@@ -188,7 +192,7 @@ __global__ void __launch_bounds__(32 * kEvalWarps)
         } else {
             for (int r = 1; r <= L; ++r) {
                 const int col = FWD ? r - 1 : L - r;
-                const bool cut = (r == L) || ((word >> ((r - 1) & 31)) & 1u);
+                const bool cut = (r == L) || brk(r - 1);
                 rp.step<FWD>(rc[col], rx[col], uint64_t(d), cut);
             }
         }

@@ -234,7 +234,7 @@ def test_profile_gen_offset_and_ragged(dc):
 
 
 # -------------------------------------------------------- timeline parity
-@pytest.mark.parametrize("L", [1, 2, 7, 16, 32, 33, 54, 65, 1024])
+@pytest.mark.parametrize("L", [1, 2, 7, 16, 32, 33, 48, 54, 64, 65, 1024])
 def test_eval_timeline_random_decisions(dc, L):
     import torch
     B = 500 + 3
