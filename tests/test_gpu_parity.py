@@ -176,6 +176,12 @@ def test_dp_batch_zero_and_single(dc):
     comp, xfer, dt = wl.random_instances(3, 1, 1, 0, 50, 0, 50)
     for d in (FWD, BWD):
         _check_direction(dc, d, comp, xfer, dt, "batch=1 L=1")
+    # one instance, and one partial tile, on every kernel family and warp count
+    for L in (16, 40, 64, 100, 200, 300):
+        for B in (1, 33):
+            comp, xfer, dt = wl.skewed_instances(11 * L + B, B, L)
+            for d in (FWD, BWD):
+                _check_direction(dc, d, comp, xfer, dt, f"batch={B} L={L}")
 
 
 def test_dp_maximum_L(dc):
