@@ -33,8 +33,8 @@
 //    kernel); the shifted values fit in signed 32 bits whenever the capped bound
 //    L*dt + sum(comp) + sum(capped xfer) is below 2^31;
 //  * value-only fill with deferred argmin, as in the short-L kernel: columns
-//    2..kKeep are written to a per-thread slot of the caller's workspace (L2
-//    resident, coalesced across the warp) and the traceback re-derives each
+//    2..8 (L <= 64) or 2..16 are written to a per-thread slot of the caller's
+//    workspace (coalesced across the warp) and the traceback re-derives each
 //    Path[m][n] as the lowest k whose candidate equals the cell. Instances whose
 //    optimum needs a deeper column, or whose values need more than 31 bits, are
 //    put on a work list that the CTA-per-instance kernel solves afterwards;
