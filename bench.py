@@ -141,6 +141,20 @@ def dp_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+def binding_roof(*roofs, **extra):
+    """The roof that binds: the one with the larger minimal time at peak, i.e. the
+    larger achieved fraction; the others follow under other_roof (one) or
+    other_roofs (several)."""
+    order = sorted(roofs, key=lambda r: -r["frac"])
+    out = dict(order[0], **extra)
+    rest = order[1:]
+    if len(rest) == 1:
+        out["other_roof"] = rest[0]
+    elif rest:
+        out["other_roofs"] = rest
+    return out
+
+
 # ------------------------------------------------------------ multi-rank
 def rank_config(base: dict, rank: int) -> dict:
     """Weak scaling: each rank solves its own `batch` distinct instances; rank r
@@ -613,10 +627,8 @@ def run_ours(args):
                 "frac": dp_gbs / hbm_peak,
                 "bytes_per_instance_direction": dp_bytes(L),
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}
-    binding, other = ((alu_roof, hbm_roof) if alu_roof["frac"] >= hbm_roof["frac"]
-                      else (hbm_roof, alu_roof))
-    roofline = dict(binding, kernel="dp_schedule (forward + backward)", traffic=traffic,
-                    other_roof=other)
+    roofline = binding_roof(alu_roof, hbm_roof, kernel="dp_schedule (forward + backward)",
+                            traffic=traffic)
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,

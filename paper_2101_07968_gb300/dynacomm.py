@@ -326,6 +326,18 @@ def greedy(direction: int, comp, xfer, dt, stream=None) -> dict:
     return out
 
 
+def shared_inputs(host_in, keys):
+    """Key -> the first key whose tensor is the same buffer (same address, size and
+    dtype); every key maps to itself when host_in is None."""
+    if host_in is None:
+        return {k: k for k in keys}
+    seen, canon = {}, {}
+    for k in keys:
+        x = host_in[k]
+        canon[k] = seen.setdefault((x.data_ptr(), x.numel(), x.dtype), k)
+    return canon
+
+
 class HostPipeline:
     """End-to-end scheduling of profiles that live in pinned host memory.
 
@@ -370,14 +382,7 @@ class HostPipeline:
         return {k: torch_empty_pinned_like(v) for k, v in self.out.items()}
 
     def _canonical(self, host_in):
-        """Input key -> the first input key holding the same host buffer."""
-        if host_in is None:
-            return {k: k for k in self.IN_KEYS}
-        seen, canon = {}, {}
-        for k in self.IN_KEYS:
-            t = host_in[k]
-            canon[k] = seen.setdefault((t.data_ptr(), t.numel(), t.dtype), k)
-        return canon
+        return shared_inputs(host_in, self.IN_KEYS)
 
     def bytes_per_run(self, host_in=None):
         """Bytes copied host->device and device->host by one run with these inputs."""
