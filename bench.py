@@ -670,7 +670,10 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     """Profiles in pinned host memory -> H2D -> forward + backward DP -> f_m of
     both -> D2H of makespans, decisions, segment counts and replays, every step,
     through dynacomm.HostPipeline (chunked: copies overlap the solves)."""
-    pipe = dc.HostPipeline(B, L, chunks=args.e2e_chunks, device=dev)
+    # pieces of at least 16,384 instances, up to 8: small batches are not worth
+    # splitting (each piece costs a few host-side calls)
+    chunks = args.e2e_chunks or max(1, min(8, B // 16384))
+    pipe = dc.HostPipeline(B, L, chunks=chunks, device=dev)
     host_in = {k: v.cpu().pin_memory() for k, v in prof.items()}
     # the gradient push of a layer moves its parameter tensor, so gt equals pt
     # (every workload here): the caller passes the one host buffer for both
@@ -698,7 +701,8 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     ms = max_over_ranks(t0.elapsed_time(t1) / steps, dev)
     return {"value": B * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps,
-            "path": f"pinned host profiles -> dynacomm.HostPipeline ({pipe.chunks} chunks, "
+            "path": f"pinned host profiles -> dynacomm.HostPipeline ({pipe.chunks} "
+                    f"piece{'s' if pipe.chunks != 1 else ''}, "
                     "copies overlapped with dc_schedule_forward/backward_batch and "
                     "dc_eval_timeline_batch) -> pinned host results",
             "inputs": "fc, pt, bc, dt; gt is the pt host buffer (equal transfer costs), "
@@ -717,7 +721,8 @@ def main(argv=None):
                         "small cases")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    p.add_argument("--e2e-chunks", type=int, default=8)
+    p.add_argument("--e2e-chunks", type=int, default=0,
+                   help="host pipeline pieces for the e2e leg (0: by batch size, up to 8)")
     p.add_argument("--lsweep", action="store_true",
                    help="scheduling time against depth L (GPU and one oracle core), one JSON line")
     p.add_argument("--compare", action="store_true",
