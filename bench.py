@@ -670,9 +670,10 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     """Profiles in pinned host memory -> H2D -> forward + backward DP -> f_m of
     both -> D2H of makespans, decisions, segment counts and replays, every step,
     through dynacomm.HostPipeline (chunked: copies overlap the solves)."""
-    # pieces of at least 16,384 instances, up to 8: small batches are not worth
-    # splitting (each piece costs a few host-side calls)
-    chunks = args.e2e_chunks or max(1, min(8, B // 16384))
+    # pieces of at least 65,536 instances, up to 8: a piece costs a few host-side
+    # calls, and its DP launch should still fill the GPU (ResNet-50: 4 pieces
+    # measured twice as fast as 8)
+    chunks = args.e2e_chunks or max(1, min(8, B // 65536))
     pipe = dc.HostPipeline(B, L, chunks=chunks, device=dev)
     host_in = {k: v.cpu().pin_memory() for k, v in prof.items()}
     # the gradient push of a layer moves its parameter tensor, so gt equals pt
@@ -722,7 +723,7 @@ def main(argv=None):
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--e2e-chunks", type=int, default=0,
-                   help="host pipeline pieces for the e2e leg (0: by batch size, up to 8)")
+                   help="host pipeline pieces for the e2e leg (0: one per 65,536 instances, 1 to 8)")
     p.add_argument("--lsweep", action="store_true",
                    help="scheduling time against depth L (GPU and one oracle core), one JSON line")
     p.add_argument("--compare", action="store_true",
