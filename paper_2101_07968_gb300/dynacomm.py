@@ -354,9 +354,12 @@ class HostPipeline:
 
     IN_KEYS = ("fc", "pt", "bc", "gt", "dt")
 
-    def __init__(self, batch: int, L: int, chunks: int = 8, device="cuda"):
+    def __init__(self, batch: int, L: int, chunks: Optional[int] = None, device="cuda"):
         import torch
         self.batch, self.L, self.W = int(batch), int(L), words(L)
+        if not chunks:  # one piece per 65,536 instances, 1 to 8: a piece costs a few
+            # host-side calls, and its DP launches should still fill the GPU
+            chunks = max(1, min(8, self.batch // 65536))
         self.chunks = max(1, min(int(chunks), self.batch))
         self.bounds = [self.batch * c // self.chunks for c in range(self.chunks + 1)]
         step = max(b - a for a, b in zip(self.bounds, self.bounds[1:]))
