@@ -670,11 +670,9 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     """Profiles in pinned host memory -> H2D -> forward + backward DP -> f_m of
     both -> D2H of makespans, decisions, segment counts and replays, every step,
     through dynacomm.HostPipeline (chunked: copies overlap the solves)."""
-    # pieces of at least 65,536 instances, up to 8: a piece costs a few host-side
-    # calls, and its DP launch should still fill the GPU (ResNet-50: 4 pieces
-    # measured twice as fast as 8)
-    chunks = args.e2e_chunks or max(1, min(8, B // 65536))
-    pipe = dc.HostPipeline(B, L, chunks=chunks, device=dev)
+    # the pipeline's default pieces: one per 65,536 instances, 1 to 8 (ResNet-50:
+    # 4 pieces measured twice as fast as 8)
+    pipe = dc.HostPipeline(B, L, chunks=args.e2e_chunks or None, device=dev)
     host_in = {k: v.cpu().pin_memory() for k, v in prof.items()}
     # the gradient push of a layer moves its parameter tensor, so gt equals pt
     # (every workload here): the caller passes the one host buffer for both
