@@ -545,8 +545,24 @@ def run_ours(args):
         if not ok:
             raise RuntimeError("timeline replay disagrees with the DP makespan")
 
+    # the same step captured once as a CUDA graph (dynacomm.StepGraph): a replay is
+    # one launch per step instead of the step's host-side calls
+    sg, graph_error = None, None
+    if not args.no_graph:
+        try:
+            sg = dc.StepGraph(cfg, device=dev)
+            for _ in range(max(args.warmup, 1)):
+                sg.replay()
+            torch.cuda.synchronize()
+            for d in (0, 1):  # same config, same results as the eager step
+                if not torch.equal(sg.sched.out[d]["makespan"], sched.out[d]["makespan"]):
+                    raise RuntimeError("graph replay disagrees with the eager step")
+        except Exception as exc:  # reported in the line; the eager timing stands
+            sg, graph_error = None, f"{type(exc).__name__}: {exc}"
+
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index if rank == 0 else -1) if rank == 0 else _Null() as clk:
         barrier()
         torch.cuda.synchronize()
@@ -556,10 +572,20 @@ def run_ours(args):
         end.record()
         torch.cuda.synchronize()
         barrier()
-    ms = start.elapsed_time(end) / max(args.steps, 1)
+        if sg is not None:
+            g0.record()
+            for s in range(args.steps):
+                sg.replay()
+            g1.record()
+            torch.cuda.synchronize()
+            barrier()
+    eager_ms = max_over_ranks(start.elapsed_time(end) / max(args.steps, 1), dev)
     seg = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])
     gen_ms, fwd_ms, bwd_ms, eval_ms = seg.mean(axis=0)
-    ms = max_over_ranks(ms, dev)
+    graph_ms = (max_over_ranks(g0.elapsed_time(g1) / max(args.steps, 1), dev)
+                if sg is not None else None)
+    ms = graph_ms if graph_ms is not None else eager_ms
+    del sg
 
     # ---- ALU roof: the DP's transition op mix, register-only, all SMs
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -647,6 +673,13 @@ def run_ours(args):
         "e2e": e2e,
         "cpu_baseline": cpu,
         "gpu_launches": launches_per_step * args.steps,
+        "timing": ("the step replayed from a CUDA graph (dynacomm.StepGraph), K replays"
+                   if graph_ms is not None else
+                   "eager launches" + (f" (graph capture failed: {graph_error})"
+                                       if graph_error else "")),
+        "eager": {"value": total / (eager_ms * 1e-3), "ms_per_step": eager_ms,
+                  "note": "the same K steps as separate library calls; breakdown_ms is "
+                          "measured on these"},
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -720,6 +753,8 @@ def main(argv=None):
                         "small cases")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-graph", action="store_true",
+                   help="time eager library calls only (no CUDA-graph replay of the step)")
     p.add_argument("--e2e-chunks", type=int, default=0,
                    help="host pipeline pieces for the e2e leg (0: one per 65,536 instances, 1 to 8)")
     p.add_argument("--lsweep", action="store_true",

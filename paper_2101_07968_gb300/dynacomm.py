@@ -326,6 +326,51 @@ def greedy(direction: int, comp, xfer, dt, stream=None) -> dict:
     return out
 
 
+class StepGraph:
+    """One whole step for a fixed config -- dc_profile_gen, the forward and backward
+    DPs and the f_m replay of both decisions -- captured once as a CUDA graph and
+    replayed. For small batches the host cost of the step's launches exceeds the
+    kernels' own time; replay() issues them as one graph launch. After each
+    replay(): prof (fc, pt, bc, gt, dt), sched.out[d] and replay_out[d] for d in
+    (FWD, BWD) hold that step's results."""
+
+    def __init__(self, cfg: dict, device="cuda"):
+        import torch
+        self.B, self.L = int(cfg["batch"]), int(cfg["L"])
+        self.keep: list = []
+        self.c = make_cfg(cfg, self.keep)
+        B, L = self.B, self.L
+        self.prof = {k: torch.empty((B, L), dtype=torch.int64, device=device)
+                     for k in ("fc", "pt", "bc", "gt")}
+        self.prof["dt"] = torch.empty(B, dtype=torch.int64, device=device)
+        self.sched = Scheduler(B, L, device=device)
+        self.replay_out = {d: torch.empty(B, dtype=torch.int64, device=device)
+                           for d in (FWD, BWD)}
+        # one eager step first: one-time setup (function attributes, occupancy
+        # queries) happens outside the capture
+        side = torch.cuda.Stream(device=device)
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            self._step()
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self._step()
+
+    def _step(self):
+        p = self.prof
+        _check(dc_profile_gen(self.c, p["fc"], p["pt"], p["bc"], p["gt"], p["dt"]),
+               "dc_profile_gen")
+        for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+            o = self.sched.run(d, p[c], p[x], p["dt"])
+            _check(dc_eval_timeline_batch(self.B, self.L, d, p[c], p[x], p["dt"], o["bits"],
+                                          self.replay_out[d]), "dc_eval_timeline_batch")
+
+    def replay(self):
+        self.graph.replay()
+
+
 def shared_inputs(host_in, keys):
     """Key -> the first key whose tensor is the same buffer (same address, size and
     dtype); every key maps to itself when host_in is None."""
