@@ -301,7 +301,7 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
 // the shifted form of the thread-per-instance kernels, all in signed 32 bits,
 // where a transition is one add-then-max and two candidates fold with one
 // 3-input min (1.5 integer-ALU instructions per transition):
-//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k] - dt,
+//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k],
 //   backward: E[m][n] = min_k max(BC[m] - (n-1)*dt + NGT[k], E[k][n-1]),
 // with G[k] = FC[L] - FC[k], Q[m] = dt + P[m] (P = transfer prefix),
 // NGT[k] = -(transfer prefix), A[m][1] = FC[L] + P[m], E[m][1] = BC[m]; U = (Q, BC)

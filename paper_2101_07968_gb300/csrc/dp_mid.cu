@@ -7,7 +7,7 @@
 // start of the cell's last transfer, so that a transition is one 32-bit
 // add-then-max and the minimum runs on 3-input mins (1.5 integer-ALU
 // instructions per transition):
-//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k] - dt,
+//   forward : B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[k] = B[k][n-1] + P[k],
 //   backward: F[m][n] - dt = min_k max(U[m] + NGT[k], F[k][n-1]),  F = X - dt - S[m],
 // with G[k] = FC[L] - FC[k], Q[m] = dt + P[m], U = BC - dt (backward),
 // NGT[k] = -(transfer prefix), A[m][1] = FC[L] + P[m], F[m][1] = BC[m]; both are

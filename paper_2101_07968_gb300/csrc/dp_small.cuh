@@ -195,7 +195,7 @@ __device__ __forceinline__ bool solve(const uint64_t (&Pc)[L + 1], const uint64_
 //
 // forward (P = transfer prefix, FC = compute prefix, G[k] = FC[L] - FC[k],
 // Q[m] = dt + P[m]): with B = X - n*dt - P[m] + G[m] (X as above) and
-// A[k] = B[k][n-1] + P[k] - dt,
+// A[k] = B[k][n-1] + P[k],
 //   B[m][n] + Q[m] = min_k max(G[k] + Q[m], A[k]),  A[m][1] = FC[L] + P[m],
 //   X[L][n] = B[L][n] + n*dt + P[L];
 // the next column's A[m] is that minimum less dt;
