@@ -260,7 +260,7 @@ def run_lsweep(args):
             gpu_s = e0.elapsed_time(e1) * 1e-3 / reps
             got = {d: {k: v.cpu().numpy() for k, v in sch.run(d, prof[c], prof[x], prof["dt"]).items()}
                    for d, (c, x) in pairs}
-            # the oracle (literal Algorithms 3 and 4) on one core; about L^3 / 3
+            # the oracle (Eq. 8 / Eq. 9 cell by cell) on one core; about L^3 / 3
             # loop iterations per instance and direction
             n_or = int(max(1, min(batch, 2e8 // (L ** 3 // 3 + 1))))
             po = oracle.profile_gen(wl.with_batch(cfg, n_or))

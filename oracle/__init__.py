@@ -1,7 +1,7 @@
 """DynaComm CPU oracle -- TEST INFRASTRUCTURE ONLY.
 
-A plain C transcription of the paper's scheduling path (Algorithm 3 / Eq. 8,
-Algorithm 4 / Eq. 9, the cost function f_m of Sec. III-B written from Eq. 1-7,
+A plain C statement of the paper's scheduling path (the recurrences Eq. 8 and
+Eq. 9 of Algorithms 3 and 4, with their choice among equal optima, the cost function f_m of Sec. III-B written from Eq. 1-7,
 brute force over the 0-1 program, the seeded profile generator standing in
 for the profiler of Sec. IV-A, and the paper's competing greedy schedulers,
 Algorithms 1 and 2), wrapped with ctypes and numpy.

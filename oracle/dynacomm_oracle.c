@@ -2,10 +2,10 @@
  * DynaComm CPU oracle: TEST INFRASTRUCTURE, not part of the product.
  * See dynacomm_oracle.h for what each function follows in the paper.
  *
- * Written to be checked by eye against the paper, not to be fast: every DP is
- * the full literal triple loop of Algorithm 3 / Algorithm 4, with the +infinity
- * entries skipped (a candidate built on F[k][n-1] = +inf can never win), and
- * every sum is a prefix-sum difference (Sec. IV-B4, "partial accumulations").
+ * Written to be checked by eye against the paper, not to be fast: each DP is
+ * its recurrence (Eq. 8, Eq. 9) evaluated cell by cell over every candidate
+ * split, with the choice among equal optima stated as a property, and every
+ * sum is a prefix-sum difference (Sec. IV-B4, "partial accumulations").
  */
 #include "dynacomm_oracle.h"
 
@@ -14,7 +14,7 @@
 #include <stdlib.h>
 #include <string.h>
 
-#define INF INT64_MAX
+#define INF INT64_MAX /* brute force: no decision seen yet */
 
 static int64_t max64(int64_t a, int64_t b) { return a > b ? a : b; }
 
@@ -33,125 +33,116 @@ static void prefix_last(int32_t L, const int64_t *v, int64_t *S)
 }
 
 /* ------------------------------------------------------------------------
- * Algorithm 3 (forward scheduling), Eq. 8:
- *   F[m][n] = min_{0<=k<m} max(F[k][n-1], n*dt + sum_{1<=l<=m} pt_l)
- *                          + sum_{k+1<=l<=m} fc_l,         1 <= n <= m <= L
- *   F[0][0] = 0, every other boundary entry +inf.
- * Ties: the strict test "if F[m][n] <= candidate: continue" keeps the lowest k;
- * the final scan keeps the lowest n. Traceback follows Path from (L, s).
- * Storage is column-major (F(m,n) at n*(L+1)+m); the loop order is the paper's.
+ * The two dynamic programs of Sec. IV-B, written from their recurrences.
+ *
+ * Take the layers in the order a direction handles them ("processing order":
+ * the forward pull starts with layer 1; the backward push starts with layer L,
+ * which is why Eq. 9 speaks of the LAST m layers). Processed layer j is layer j
+ * forward and layer L+1-j backward. C(m) and T(m) are the compute and transfer
+ * costs summed over the first m processed layers (prefix sums, Sec. IV-B4).
+ * X(m, n) is the least finishing time of the first m processed layers when
+ * their transfer is cut into exactly n segments, the last one holding
+ * processed layers k+1..m:
+ *
+ *   forward,  Eq. 8:  X(m, n) = min_k max(X(k, n-1), n*dt + T(m)) + C(m) - C(k)
+ *     (the n-th pull has arrived at n*dt + T(m); layers k+1..m then compute
+ *      after the first k layers are done);
+ *   backward, Eq. 9:  X(m, n) = min_k max(X(k, n-1), C(m)) + dt + T(m) - T(k)
+ *     (the n-th push waits for the backward compute of its layers and for the
+ *      previous push, then carries dt plus the gradients of layers k+1..m).
+ *
+ * X(0, 0) = 0 and X(k, n-1) exists only when 0 layers are cut into 0 segments
+ * or 1 <= n-1 <= k; that is reading R1 (the paper's +infinity entries never
+ * win, so they are simply not candidates).
+ *
+ * Which of several optima is returned is fixed by the paper's algorithms
+ * (reading R3), and stated here as properties:
+ *   - Path(m, n) is the SMALLEST k attaining the minimum (their strict
+ *     improvement test keeps the first minimiser as k grows);
+ *   - the segment count s is the SMALLEST n attaining min_n X(L, n);
+ *   - the decision is read from state (L, s) by stepping (m, n) ->
+ *     (Path(m, n), n-1) down to (0, 0); every k reached with 1 <= k <= L-1
+ *     enables the position after processed layer k: p_k forward (a new pull
+ *     from layer k+1), g_k backward (a new push after the last k layers,
+ *     between layers L-k and L-k+1; reading R4, which Algorithm 4's index
+ *     conversion expresses).
+ * Storage: X and Path are (L+1) x (L+1), column n contiguous (n*(L+1) + m).
  * ---------------------------------------------------------------------- */
+
+/* can the first k processed layers be cut into exactly n segments? */
+static int split_exists(int32_t k, int32_t n) { return n == 0 ? k == 0 : (n >= 1 && n <= k); }
+
+static int64_t segment_end(int32_t dir, int64_t before, int32_t m, int32_t n, int32_t k,
+                           const int64_t *C, const int64_t *T, int64_t dt)
+{
+    if (dir == 0) /* Eq. 8 */
+        return max64(before, (int64_t)n * dt + T[m]) + (C[m] - C[k]);
+    return max64(before, C[m]) + dt + (T[m] - T[k]); /* Eq. 9 */
+}
+
+/* comp/xfer hold layer l at index l-1 (l = 1..L), in layer order. Writes the
+ * decision d[0..L] (entries 1..L-1 used) and *nseg; returns min_n X(L, n). */
+static int64_t solve_dp(int32_t dir, int32_t L, const int64_t *comp, const int64_t *xfer,
+                        int64_t dt, uint8_t *d, int32_t *nseg)
+{
+    const size_t W = (size_t)L + 1;
+    int64_t *X = (int64_t *)malloc(W * W * sizeof(int64_t));
+    int32_t *Path = (int32_t *)malloc(W * W * sizeof(int32_t));
+    int64_t *C = (int64_t *)malloc(W * sizeof(int64_t));
+    int64_t *T = (int64_t *)malloc(W * sizeof(int64_t));
+    if (dir == 0) {
+        prefix_first(L, comp, C);
+        prefix_first(L, xfer, T);
+    } else {
+        prefix_last(L, comp, C);
+        prefix_last(L, xfer, T);
+    }
+    X[0] = 0; /* X(0, 0) */
+    for (int32_t n = 1; n <= L; n++)      /* column by column: X(., n) needs X(., n-1) */
+        for (int32_t m = n; m <= L; m++) { /* cells that exist: n <= m */
+            int64_t best = 0;
+            int32_t arg = -1;
+            for (int32_t k = n - 1; k <= m - 1; k++) {
+                if (!split_exists(k, n - 1)) continue;
+                int64_t c = segment_end(dir, X[(size_t)(n - 1) * W + (size_t)k], m, n, k, C, T, dt);
+                if (arg < 0 || c < best) { /* ties keep the smaller k */
+                    best = c;
+                    arg = k;
+                }
+            }
+            X[(size_t)n * W + (size_t)m] = best;
+            Path[(size_t)n * W + (size_t)m] = arg;
+        }
+    int32_t s = 1;
+    for (int32_t n = 2; n <= L; n++) /* ties keep the smaller n */
+        if (X[(size_t)n * W + (size_t)L] < X[(size_t)s * W + (size_t)L]) s = n;
+    const int64_t opt = X[(size_t)s * W + (size_t)L];
+    memset(d, 0, W);
+    for (int32_t m = L, n = s; n > 0; n--) {
+        const int32_t k = Path[(size_t)n * W + (size_t)m];
+        if (k >= 1 && k <= L - 1) d[k] = 1;
+        m = k;
+    }
+    *nseg = s;
+    free(X);
+    free(Path);
+    free(C);
+    free(T);
+    return opt;
+}
+
+/* Forward (Eq. 8, the problem of Algorithm 3): comp = fc, xfer = pt. */
 int64_t orc_dp_forward(int32_t L, const int64_t *pt, const int64_t *fc, int64_t dt,
                        uint8_t *p, int32_t *nseg)
 {
-    const size_t W = (size_t)L + 1;
-    int64_t *F = (int64_t *)malloc(W * W * sizeof(int64_t));
-    int32_t *Path = (int32_t *)malloc(W * W * sizeof(int32_t));
-    int64_t *P = (int64_t *)malloc(W * sizeof(int64_t));
-    int64_t *FC = (int64_t *)malloc(W * sizeof(int64_t));
-#define F_(m, n) F[(size_t)(n) * W + (size_t)(m)]
-#define PATH_(m, n) Path[(size_t)(n) * W + (size_t)(m)]
-    prefix_first(L, pt, P);
-    prefix_first(L, fc, FC);
-    for (int32_t m = 0; m <= L; m++)
-        for (int32_t n = 0; n <= L; n++) {
-            F_(m, n) = INF;
-            PATH_(m, n) = -1;
-        }
-    F_(0, 0) = 0;
-    for (int32_t m = 1; m <= L; m++)
-        for (int32_t n = 1; n <= m; n++)
-            for (int32_t k = 0; k <= m - 1; k++) {
-                if (F_(k, n - 1) == INF) continue; /* +inf never improves */
-                int64_t t_lst = max64(F_(k, n - 1), (int64_t)n * dt + P[m]);
-                int64_t cand = t_lst + (FC[m] - FC[k]);
-                if (F_(m, n) <= cand) continue;
-                F_(m, n) = cand;
-                PATH_(m, n) = k;
-            }
-    int64_t t_fwd = INF;
-    int32_t s = -1;
-    for (int32_t k = 1; k <= L; k++) {
-        if (t_fwd <= F_(L, k)) continue;
-        t_fwd = F_(L, k);
-        s = k;
-    }
-    memset(p, 0, (size_t)L + 1);
-    int32_t cl = L;
-    for (int32_t k = 1; k <= s; k++) {
-        int32_t tmp = PATH_(cl, s - k + 1);
-        if (1 <= tmp && tmp <= L - 1) p[tmp] = 1;
-        cl = tmp;
-    }
-    *nseg = s;
-#undef F_
-#undef PATH_
-    free(F);
-    free(Path);
-    free(P);
-    free(FC);
-    return t_fwd;
+    return solve_dp(0, L, fc, pt, dt, p, nseg);
 }
 
-/* ------------------------------------------------------------------------
- * Algorithm 4 (backward scheduling), Eq. 9:
- *   B[m][n] = min_{0<=k<m} max(B[k][n-1], sum_{L-m+1<=l<=L} bc_l) + dt
- *                          + sum_{L-m+1<=l<=L-k} gt_l,     1 <= n <= m <= L
- * m counts the LAST m layers. The final scan reads B[L][k] (the listing prints
- * F[L][k] there, a typo: only B exists in this algorithm). Traceback uses the
- * listing's index conversion Path[L - cl + 1][.] with cl = L - tmp + 1.
- * ---------------------------------------------------------------------- */
+/* Backward (Eq. 9, the problem of Algorithm 4): comp = bc, xfer = gt. */
 int64_t orc_dp_backward(int32_t L, const int64_t *bc, const int64_t *gt, int64_t dt,
                         uint8_t *g, int32_t *nseg)
 {
-    const size_t W = (size_t)L + 1;
-    int64_t *B = (int64_t *)malloc(W * W * sizeof(int64_t));
-    int32_t *Path = (int32_t *)malloc(W * W * sizeof(int32_t));
-    int64_t *SBC = (int64_t *)malloc(W * sizeof(int64_t));
-    int64_t *SGT = (int64_t *)malloc(W * sizeof(int64_t));
-#define B_(m, n) B[(size_t)(n) * W + (size_t)(m)]
-#define PATH_(m, n) Path[(size_t)(n) * W + (size_t)(m)]
-    prefix_last(L, bc, SBC);
-    prefix_last(L, gt, SGT);
-    for (int32_t m = 0; m <= L; m++)
-        for (int32_t n = 0; n <= L; n++) {
-            B_(m, n) = INF;
-            PATH_(m, n) = -1;
-        }
-    B_(0, 0) = 0;
-    for (int32_t m = 1; m <= L; m++)
-        for (int32_t n = 1; n <= m; n++)
-            for (int32_t k = 0; k <= m - 1; k++) {
-                if (B_(k, n - 1) == INF) continue;
-                int64_t t_lst = max64(B_(k, n - 1), SBC[m]);
-                /* sum_{L-m+1 <= l <= L-k} gt_l = SGT[m] - SGT[k] */
-                int64_t cand = t_lst + dt + (SGT[m] - SGT[k]);
-                if (B_(m, n) <= cand) continue;
-                B_(m, n) = cand;
-                PATH_(m, n) = k;
-            }
-    int64_t t_bwd = INF;
-    int32_t s = -1;
-    for (int32_t k = 1; k <= L; k++) {
-        if (t_bwd <= B_(L, k)) continue;
-        t_bwd = B_(L, k);
-        s = k;
-    }
-    memset(g, 0, (size_t)L + 1);
-    int32_t cl = 1;
-    for (int32_t k = 1; k <= s; k++) {
-        int32_t tmp = PATH_(L - cl + 1, s - k + 1);
-        if (1 <= tmp && tmp <= L - 1) g[tmp] = 1;
-        cl = L - tmp + 1;
-    }
-    *nseg = s;
-#undef B_
-#undef PATH_
-    free(B);
-    free(Path);
-    free(SBC);
-    free(SGT);
-    return t_bwd;
+    return solve_dp(1, L, bc, gt, dt, g, nseg);
 }
 
 /* ------------------------------------------------------------------------

@@ -1,11 +1,13 @@
 /*
  * DynaComm CPU oracle: TEST INFRASTRUCTURE, not part of the product.
  *
- * A plain, slow, single-threaded C transcription of what the DynaComm scheduling
+ * A plain, slow, single-threaded C statement of what the DynaComm scheduling
  * path computes (Cai et al., "DynaComm: Accelerating Distributed CNN Training
  * between Edges and Clouds through Dynamic Communication Scheduling"):
- *   - the forward DP, Eq. 8 filled in the loop order of Algorithm 3,
- *   - the backward DP, Eq. 9 filled in the loop order of Algorithm 4,
+ *   - the forward DP, Eq. 8 evaluated cell by cell (the problem Algorithm 3 solves),
+ *   - the backward DP, Eq. 9 evaluated cell by cell (the problem of Algorithm 4),
+ *     both returning the optimum Algorithms 3/4 return among equal ones: the
+ *     lowest split index per cell, the lowest segment count overall,
  *   - the cost measurement f_m of Sec. III-B, written as an event replay of the
  *     partial orders Eq. 1-7,
  *   - brute force over all 2^(L-1) decisions (Sec. III-B, the O(L 2^L) search),

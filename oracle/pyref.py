@@ -1,89 +1,86 @@
-"""Second, independent transcription of Algorithms 3 and 4 in pure Python.
+"""A second, independent oracle for the two dynamic programs, in pure Python.
 
 TEST INFRASTRUCTURE ONLY (same import rule as the C oracle). It exists to
-cross-check the C oracle on tie-heavy small inputs, where the exact boundaries
-depend on the listings' tie-break rules rather than on the optimum alone. Sums
-are taken directly over their index ranges as Eq. 8 / Eq. 9 print them, with no
-prefix arrays, so the two transcriptions share neither code nor structure.
+cross-check the C oracle on small, tie-heavy inputs, where the exact boundaries
+depend on which of several optima is returned rather than on the optimum alone.
+
+It is written differently from the C oracle on purpose: top-down, as a
+memoised recursion over sub-problems (m layers, n segments) of Sec. IV-B1, with
+every sum taken directly over its index range as Eq. 8 / Eq. 9 print it (no
+prefix arrays), and the choice among equal optima made by comparing (value,
+index) pairs: the smallest value wins and, on a tie, the smallest index -- the
+lowest split k within a cell and the lowest segment count n overall, which is
+what the paper's algorithms return (their improvement tests are strict).
 Use for L up to about 30.
 """
 from __future__ import annotations
 
-INF = float("inf")
+import sys
+from functools import lru_cache
+
+
+def _solve(L, last_segment_end):
+    """Least finishing time over cuts of all L processed layers, the cut that
+    attains it and its segment count. last_segment_end(m, n, k, before) is the
+    finishing time of processed layers k+1..m sent as the n-th segment, once the
+    first k layers finished (in n-1 segments) at `before`."""
+    sys.setrecursionlimit(max(sys.getrecursionlimit(), 10 * L + 100))
+
+    @lru_cache(maxsize=None)
+    def best(m, n):
+        """(X(m, n), lowest minimising k), or None when m layers cannot form n segments."""
+        if n == 0:
+            return (0, None) if m == 0 else None
+        if m < n:
+            return None
+        options = []
+        for k in range(m):  # the n-th segment holds processed layers k+1..m
+            sub = best(k, n - 1)
+            if sub is not None:
+                options.append((last_segment_end(m, n, k, sub[0]), k))
+        return min(options)
+
+    value, s = min((best(L, n)[0], n) for n in range(1, L + 1))
+    cut = [0] * (L + 1)
+    m, n = L, s
+    while n > 0:
+        k = best(m, n)[1]
+        if 1 <= k <= L - 1:
+            cut[k] = 1
+        m, n = k, n - 1
+    return value, cut, s
 
 
 def forward(pt, fc, dt):
-    """Algorithm 3 with Eq. 8. pt, fc: per-layer lists (layer l at index l-1).
+    """Eq. 8. pt, fc: per-layer lists (layer l at index l-1).
 
-    Returns (T_forward, p as a list of L+1 ints, number of enabled positions)."""
+    Returns (T_forward, p as a list of L+1 ints, number of segments)."""
     L = len(pt)
-    F = [[INF] * (L + 1) for _ in range(L + 1)]
-    path = [[-1] * (L + 1) for _ in range(L + 1)]
-    F[0][0] = 0
-    for m in range(1, L + 1):
-        for n in range(1, m + 1):
-            for k in range(0, m):
-                if F[k][n - 1] == INF:
-                    continue
-                pull_done = n * dt + sum(pt[l - 1] for l in range(1, m + 1))
-                t_lst = max(F[k][n - 1], pull_done)
-                cost = t_lst + sum(fc[l - 1] for l in range(k + 1, m + 1))
-                if F[m][n] <= cost:
-                    continue
-                F[m][n] = cost
-                path[m][n] = k
-    best, steps = INF, -1
-    for k in range(1, L + 1):
-        if best <= F[L][k]:
-            continue
-        best, steps = F[L][k], k
-    p = [0] * (L + 1)
-    cur = L
-    for k in range(1, steps + 1):
-        tmp = path[cur][steps - k + 1]
-        if 1 <= tmp <= L - 1:
-            p[tmp] = 1
-        cur = tmp
-    return best, p, steps
+
+    def end(m, n, k, before):
+        arrived = n * dt + sum(pt[l - 1] for l in range(1, m + 1))
+        return max(before, arrived) + sum(fc[l - 1] for l in range(k + 1, m + 1))
+
+    return _solve(L, end)
 
 
 def backward(bc, gt, dt):
-    """Algorithm 4 with Eq. 9. bc, gt: per-layer lists in layer order 1..L."""
+    """Eq. 9. bc, gt: per-layer lists in layer order 1..L; sub-problems hold the
+    LAST m layers, so g[k] = 1 is a break after the last k layers."""
     L = len(bc)
-    B = [[INF] * (L + 1) for _ in range(L + 1)]
-    path = [[-1] * (L + 1) for _ in range(L + 1)]
-    B[0][0] = 0
-    for m in range(1, L + 1):
-        for n in range(1, m + 1):
-            for k in range(0, m):
-                if B[k][n - 1] == INF:
-                    continue
-                comp_done = sum(bc[l - 1] for l in range(L - m + 1, L + 1))
-                t_lst = max(B[k][n - 1], comp_done)
-                cost = t_lst + dt + sum(gt[l - 1] for l in range(L - m + 1, L - k + 1))
-                if B[m][n] <= cost:
-                    continue
-                B[m][n] = cost
-                path[m][n] = k
-    best, steps = INF, -1
-    for k in range(1, L + 1):
-        if best <= B[L][k]:
-            continue
-        best, steps = B[L][k], k
-    g = [0] * (L + 1)
-    cl = 1
-    for k in range(1, steps + 1):
-        tmp = path[L - cl + 1][steps - k + 1]
-        if 1 <= tmp <= L - 1:
-            g[tmp] = 1
-        cl = L - tmp + 1
-    return best, g, steps
+
+    def end(m, n, k, before):
+        computed = sum(bc[l - 1] for l in range(L - m + 1, L + 1))
+        pushed = sum(gt[l - 1] for l in range(L - m + 1, L - k + 1))
+        return max(before, computed) + dt + pushed
+
+    return _solve(L, end)
 
 
 # ---------------------------------------------------------------------------
-# The competing greedy schedulers (Algorithms 1 and 2), transcribed again with
+# The competing greedy schedulers (Algorithms 1 and 2), written again with
 # explicit candidate lists and key tuples. Readings (same as the C oracle's
-# G1-G5): ties keep the first candidate of the listing's enumeration; an empty
+# G1-G5): ties keep the first candidate in enumeration order; an empty
 # Options set takes the largest slack; Algorithm 1's first pair orders S2 by
 # (max first compute, min first transfer, min slack, enumeration order); the
 # estimated total execution time of Algorithm 2 is the backward makespan.

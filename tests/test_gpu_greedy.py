@@ -1,9 +1,9 @@
 """GPU greedy schedulers (Algorithm 1 forward, Algorithm 2 backward) against the
-oracle's literal transcriptions, through the C ABI: every decision word and
+oracle's greedy schedulers, through the C ABI: every decision word and
 every makespan bit-exact, faults included.
 
-The oracle enumerates every pair and position with direct range sums (Algorithm
-2 costs O(L^4) there), so the CNN batches are checked on samples and the
+The oracle enumerates every pair and position (Algorithm 2 costs O(L^3) there,
+plus a replay per candidate), so the CNN batches are checked on samples and the
 decisions of the whole batch are replayed instead.
 """
 import os

@@ -1,9 +1,10 @@
 """Pins of the oracle's competing greedy schedulers (Algorithms 1 and 2).
 
 The greedy algorithms have no closed form; they are pinned by hand-worked
-examples (tests/golden/greedy_worked.txt, derived from the listings' steps), by
-a second, independent transcription (oracle/pyref.py, explicit candidate lists
-and its own replay), by special cases whose outcome the listings fix, and by
+examples (tests/golden/greedy_worked.txt, worked by hand from the greedy rules
+of Sec. II-C), by a second, independent oracle (oracle/pyref.py, explicit
+candidate lists and its own replay), by special cases whose outcome the
+algorithms fix, and by
 the optimality of the DP (no greedy decision beats Algorithms 3/4).
 """
 import os
@@ -42,7 +43,7 @@ def test_worked_examples(case):
 
 @pytest.mark.parametrize("L", range(1, 11))
 @pytest.mark.parametrize("kind", ["tie", "uni", "skew"])
-def test_two_transcriptions_agree(L, kind):
+def test_two_oracles_agree(L, kind):
     gen = {"tie": wl.tie_heavy_instances, "uni": wl.random_instances,
            "skew": wl.skewed_instances}[kind]
     comp, xfer, dt = gen(97 * L + len(kind), 120, L)
@@ -66,7 +67,7 @@ def _pack(d, L):
 
 
 def test_short_models():
-    """L = 1: the single segment; L = 2: both listings end at layer by layer."""
+    """L = 1: the single segment; L = 2: both algorithms end at layer by layer."""
     assert list(oracle.greedy_forward([5], [7], 3)) == [0, 0]
     assert list(oracle.greedy_backward([5], [7], 3)) == [0, 0]
     comp, xfer, dt = wl.random_instances(4, 200, 2, 0, 1000, 0, 1000)

@@ -47,7 +47,7 @@ def test_dp_equals_brute_force(orc, kind, direction):
         assert orc.replay(direction, comp, xfer, dt, d) == v
 
 
-def _literal_traceback_by_enumeration(orc, direction, comp, xfer, dt):
+def _traceback_by_enumeration(orc, direction, comp, xfer, dt):
     """The decision Algorithm 3/4 returns, derived without the recurrence:
     opt(m, n) comes from enumerating every decision of the sub-problem; the
     traceback starts at the fewest-segment optimum (L, s) and from (m, n) steps
@@ -84,7 +84,7 @@ def test_traceback_tie_break_by_enumeration(orc, direction):
     """Pins the exact boundaries (not only the optimum) on tie-heavy inputs."""
     for comp, xfer, dt in _cases(31 + direction, 300, 8, "tie"):
         v, d, s = orc.dp(direction, comp, xfer, dt)
-        bv, bd, bs = _literal_traceback_by_enumeration(orc, direction, comp, xfer, dt)
+        bv, bd, bs = _traceback_by_enumeration(orc, direction, comp, xfer, dt)
         assert (v, s) == (bv, bs)
         assert list(d) == bd, (comp, xfer, dt)
 
@@ -115,9 +115,9 @@ def test_subproblem_values_enumeration_consistency(orc):
                     assert min(cands) == X[(m, n)]
 
 
-# ------------------------------------------------------------ second transcription
+# ------------------------------------------------------------ second oracle
 @pytest.mark.parametrize("direction", [FWD, BWD])
-def test_python_transcription_agrees(orc, direction):
+def test_python_oracle_agrees(orc, direction):
     for kind in ("tie", "uni"):
         for comp, xfer, dt in _cases(51 + direction, 150, 10, kind):
             v, d, s = orc.dp(direction, comp, xfer, dt)
@@ -291,6 +291,64 @@ def test_loguniform_distribution(orc):
         assert abs(frac - 1 / 3) < 0.02
     assert orc.loguniform(lo, hi, 0) == lo
     assert orc.loguniform(lo, hi, 2**64 - 1) <= hi
+
+
+def test_loguniform_knots_hand_worked(orc):
+    """Knots worked by hand from the definition of the log-uniform draw
+    (tests/golden/loguniform_knots.txt): T(256) is the geometric mean, T(128)
+    and T(384) the quarter points. A draw with top 9 bits j and zero fraction
+    bits returns T(j)."""
+    for row in read_golden("loguniform_knots.txt"):
+        lo, hi, j, t = row[:4]  # the rest of the row is the derivation
+        assert orc.loguniform(int(lo), int(hi), int(j) << 55) == int(t), (lo, hi, j)
+
+
+_LOGU_RANGES = [(1_000, 100_000), (1_000, 1_000_000), (5_000, 200_000),
+                (1_000, 10_000_000), (1_000_000, 10_000_000_000)]
+
+
+def _exact_knots(lo, hi):
+    """T(j) = lo * (hi/lo)^(j/512) for j = 0..512 at 50 significant digits,
+    rounded half away from zero; None where the value lies within 1e-6 of a
+    half (there a double-precision evaluation may round either way)."""
+    from decimal import ROUND_HALF_UP, Decimal, localcontext
+    out = []
+    with localcontext() as ctx:
+        ctx.prec = 50
+        ratio = Decimal(hi) / Decimal(lo)
+        for j in range(513):
+            v = Decimal(lo) * ratio ** (Decimal(j) / Decimal(512))
+            frac = v - int(v)
+            near_half = abs(frac - Decimal("0.5")) < Decimal("1e-6")
+            out.append(None if near_half else int(v.quantize(Decimal(1), rounding=ROUND_HALF_UP)))
+    return out
+
+
+@pytest.mark.parametrize("lo,hi", _LOGU_RANGES)
+def test_loguniform_matches_its_definition(orc, lo, hi):
+    """Every knot of the five workloads' ranges, and full draws (knot plus the
+    linear step between knots j and j+1 scaled by the 32 fraction bits), against
+    the definition evaluated in 50-digit decimal arithmetic. A change of the
+    knot spacing (say j/511 for j/512), of the bit fields or of the rounding
+    fails here."""
+    T = _exact_knots(lo, hi)
+    assert T[0] == lo and T[512] == hi
+    skipped = 0
+    for j in range(512):
+        if T[j] is None:
+            skipped += 1
+            continue
+        assert orc.loguniform(lo, hi, j << 55) == T[j], (lo, hi, j)
+    assert skipped <= 2
+    rng = np.random.default_rng(lo ^ hi)
+    for _ in range(3000):
+        r = int(rng.integers(0, 2**63)) * 2 + int(rng.integers(0, 2))
+        j, f = r >> 55, (r >> 23) & 0xFFFFFFFF
+        if T[j] is None or T[j + 1] is None:
+            continue
+        assert orc.loguniform(lo, hi, r) == T[j] + (((T[j + 1] - T[j]) * f) >> 32), (lo, hi, r)
+    # the top knot: j = 511 with every fraction bit set reaches hi - 1 (hi - T(511) >= 1)
+    assert orc.loguniform(lo, hi, (511 << 55) | (0xFFFFFFFF << 23)) == hi - 1
 
 
 @pytest.mark.parametrize("name", ["tiny", "alexnet", "vgg16", "resnet50"])
