@@ -1,7 +1,8 @@
 """Build libdynacomm.so (sm_103a) in-tree with nvcc; no CMake, no torch extension.
 
 Each .cu under csrc/ is compiled in parallel, then linked into one shared
-library with the static CUDA runtime. ``python -m paper_2101_07968_gb300.build``
+library against the shared CUDA runtime (libcudart.so.13, the copy torch
+loads when it is already in the process). ``python -m paper_2101_07968_gb300.build``
 builds it; ``build(verbose=True)`` also prints ptxas register/spill reports.
 """
 from __future__ import annotations

@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <mutex>
 
 #include <cuda_runtime.h>
 
@@ -73,6 +74,40 @@ struct Workspace {
     {
         return group_tables_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
     }
+};
+
+// A per-device launch fact (resident CTAs per SM of a kernel, the SM count),
+// found once per device by the first call that needs it; `lookup` may also
+// raise a kernel's shared-memory limit on the way. Thread-safe: lookups run
+// under the cache's mutex, so host threads that launch at once do not race,
+// and each device ordinal keeps its own value. A context re-created after
+// cudaDeviceReset keeps these numbers (they describe the device); a kernel
+// attribute raised in the old context is gone, and a launch that needed it
+// then fails with a CUDA error instead of running.
+constexpr int kMaxDevices = 64;
+class DeviceCache {
+public:
+    template <typename F>
+    cudaError_t get(int &out, F &&lookup)
+    {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+        std::lock_guard<std::mutex> lock(mu_);
+        if (value_[dev] <= 0) {
+            int v = 0;
+            e = lookup(v);
+            if (e != cudaSuccess) return e;
+            value_[dev] = v > 0 ? v : 1;
+        }
+        out = value_[dev];
+        return cudaSuccess;
+    }
+
+private:
+    std::mutex mu_;
+    int value_[kMaxDevices] = {};
 };
 
 // L*dt + sum(comp) + sum(xfer) >= 2^52, for inputs already known to be

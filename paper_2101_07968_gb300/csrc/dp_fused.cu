@@ -141,14 +141,14 @@ cudaError_t launch_fused_list(const GenParams &g, const GenTables *t, const Fuse
                               cudaStream_t stream)
 {
     using K64 = Small<L, uint64_t, L>;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(fused_list_kernel<L, FWD>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             K64::kTableBytes);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    static DeviceCache attr;  // the list kernel's shared-memory limit, raised once per device
+    int done = 0;
+    cudaError_t ae = attr.get(done, [](int &v) {
+        v = 1;
+        return cudaFuncSetAttribute(fused_list_kernel<L, FWD>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, K64::kTableBytes);
+    });
+    if (ae != cudaSuccess) return ae;
     int64_t lgrid = (g.batch + 31) / 32;
     if (lgrid > int64_t(sm_count()) * 4) lgrid = int64_t(sm_count()) * 4;
     cudaLaunchConfig_t lc = {};
@@ -169,18 +169,17 @@ cudaError_t launch_fused_dir(const GenParams &g, const GenTables *t, const Fused
                              cudaStream_t stream)
 {
     using K32 = Small<L, uint32_t, kKeepCols>;
-    static int per_sm = 0;
-    if (per_sm == 0) {
+    static DeviceCache resident;  // single-warp CTAs of the fused kernel per SM
+    int per_sm = 0;
+    cudaError_t le = resident.get(per_sm, [](int &n) {
         cudaError_t e = cudaFuncSetAttribute(fused_dense_kernel<L, FWD>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              K32::kWarpBytes);
         if (e != cudaSuccess) return e;
-        int n = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fused_dense_kernel<L, FWD>, 32,
-                                                          K32::kWarpBytes);
-        if (e != cudaSuccess) return e;
-        per_sm = n > 0 ? n : 1;
-    }
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fused_dense_kernel<L, FWD>, 32,
+                                                             K32::kWarpBytes);
+    });
+    if (le != cudaSuccess) return le;
     const int64_t tiles = (g.batch + 31) / 32;
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;

@@ -419,14 +419,15 @@ cudaError_t launch_mid_nw(int64_t batch, int L, const int64_t *comp, const int64
                           uint32_t *list, uint32_t *tb, cudaStream_t stream)
 {
     const size_t smem = size_t(3) * (L + 1) * 32 * 4;
-    static bool attr = false;
-    if (!attr) {
+    static DeviceCache attr;  // the kernel's shared-memory limit, raised once per device
+    int done = 0;
+    const cudaError_t ae = attr.get(done, [](int &v) {
         const int most = 3 * (kMidLMax + 1) * 32 * 4;
-        cudaError_t e = cudaFuncSetAttribute(mid_kernel<FWD, NW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+        v = 1;
+        return cudaFuncSetAttribute(mid_kernel<FWD, NW>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+    });
+    if (ae != cudaSuccess) return ae;
     const int64_t slots = mid_slots(batch, L);
     const int64_t grid = slots / 32;
     mid_kernel<FWD, NW><<<unsigned(grid), 32 * NW, smem, stream>>>(

@@ -139,19 +139,19 @@ __global__ void __launch_bounds__(32)
     }
 }
 
-int g_sm_count = 0;
-
 }  // namespace
 
 int sm_count()
 {
-    if (g_sm_count == 0) {
+    static DeviceCache sms;
+    int n = 0;
+    const cudaError_t e = sms.get(n, [](int &v) {
         int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sm_count, cudaDevAttrMultiProcessorCount, dev);
-        if (g_sm_count <= 0) g_sm_count = 152;
-    }
-    return g_sm_count;
+        cudaError_t r = cudaGetDevice(&dev);
+        if (r == cudaSuccess) r = cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        return r;
+    });
+    return e == cudaSuccess ? n : 152;
 }
 
 namespace {
@@ -164,8 +164,9 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
 {
     using K32 = Small<L, uint32_t, kKeepCols>;
     using K64 = Small<L, uint64_t, L>;
-    static int per_sm = 0;  // resident single-warp CTAs per SM for the dense kernel
-    if (per_sm == 0) {
+    static DeviceCache resident;  // single-warp CTAs of the dense kernel per SM
+    int per_sm = 0;
+    cudaError_t le = resident.get(per_sm, [](int &n) {
         cudaError_t e = cudaFuncSetAttribute(small_dense_kernel<L, FWD>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              K32::kWarpBytes);
@@ -173,12 +174,10 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
         e = cudaFuncSetAttribute(small_list_kernel<L, FWD>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, K64::kTableBytes);
         if (e != cudaSuccess) return e;
-        int n = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, small_dense_kernel<L, FWD>, 32,
-                                                          K32::kWarpBytes);
-        if (e != cudaSuccess) return e;
-        per_sm = n > 0 ? n : 1;
-    }
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, small_dense_kernel<L, FWD>, 32,
+                                                             K32::kWarpBytes);
+    });
+    if (le != cudaSuccess) return le;
     const int64_t tiles = (batch + 31) / 32;
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;

@@ -319,16 +319,16 @@ cudaError_t launch_small_eval(int64_t batch, const int64_t *comp, const int64_t 
 {
     constexpr int kStride = (L % 2 == 1) ? L : (L % 4 == 2 ? L : L + 2);
     constexpr int smem = kEvalWarps * 2 * 32 * kStride * 8;
-    static int per_sm = 0;
-    if (per_sm == 0) {
+    static DeviceCache resident;  // CTAs of the replay kernel per SM
+    int per_sm = 0;
+    const cudaError_t le = resident.get(per_sm, [](int &n) {
         cudaError_t e = cudaFuncSetAttribute(eval_small_kernel<L, FWD>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e == cudaSuccess)
-            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, eval_small_kernel<L, FWD>,
-                                                              32 * kEvalWarps, smem);
         if (e != cudaSuccess) return e;
-        if (per_sm < 1) per_sm = 1;
-    }
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, eval_small_kernel<L, FWD>,
+                                                             32 * kEvalWarps, smem);
+    });
+    if (le != cudaSuccess) return le;
     int64_t blocks = ((batch + 31) / 32 + kEvalWarps - 1) / kEvalWarps;
     if (blocks > int64_t(sm_count()) * per_sm) blocks = int64_t(sm_count()) * per_sm;
     eval_small_kernel<L, FWD><<<unsigned(blocks), 32 * kEvalWarps, smem, stream>>>(
@@ -363,29 +363,30 @@ cudaError_t launch_eval(bool forward, int64_t batch, int L, const int64_t *comp,
         const int stride = eval_stride(L);
         const size_t smem = size_t(kEvalWarps) * 2 * 32 * stride * 8;
         const bool pairs = ((reinterpret_cast<uintptr_t>(comp) | reinterpret_cast<uintptr_t>(xfer)) & 15u) == 0;
-        static bool attr_set = false;  // up to 69.6 KB at L = 32: above the 48 KB default
-        if (!attr_set) {
+        // up to 69.6 KB at L = 32: above the 48 KB default
+        static DeviceCache attr;
+        int done = 0;
+        cudaError_t ae = attr.get(done, [](int &v) {
             const int most = kEvalWarps * 2 * 32 * (kStagedLMax + 2) * 8;
+            v = 1;
             cudaError_t e = cudaFuncSetAttribute(
                 eval_staged_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(eval_staged_kernel<false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, most);
             if (e != cudaSuccess) return e;
-            attr_set = true;
-        }
+            return cudaFuncSetAttribute(eval_staged_kernel<false>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        });
+        if (ae != cudaSuccess) return ae;
         // persistent warps: one resident wave, each warp walking tiles (and
-        // prefetching its next one)
-        static int resident[kStagedLMax + 1][2];
-        int &per_sm = resident[L][forward ? 1 : 0];
-        if (per_sm == 0) {
-            cudaError_t e = forward ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                                          &per_sm, eval_staged_kernel<true>, 32 * kEvalWarps, smem)
-                                    : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                                          &per_sm, eval_staged_kernel<false>, 32 * kEvalWarps, smem);
-            if (e != cudaSuccess) return e;
-            if (per_sm < 1) per_sm = 1;
-        }
+        // prefetching its next one); resident CTAs per SM by L and direction
+        static DeviceCache resident[kStagedLMax + 1][2];
+        int per_sm = 0;
+        ae = resident[L][forward ? 1 : 0].get(per_sm, [&](int &n) {
+            return forward ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                 &n, eval_staged_kernel<true>, 32 * kEvalWarps, smem)
+                           : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                 &n, eval_staged_kernel<false>, 32 * kEvalWarps, smem);
+        });
+        if (ae != cudaSuccess) return ae;
         int64_t blocks = ((batch + 31) / 32 + kEvalWarps - 1) / kEvalWarps;
         if (blocks > int64_t(sm_count()) * per_sm) blocks = int64_t(sm_count()) * per_sm;
         if (forward)
