@@ -216,9 +216,11 @@ dc_status dc_eval_timeline_batch(int64_t batch, int32_t L, int32_t dir, const in
  * between a gradient push and the next pull, where a cudaMalloc that can
  * synchronise the device is not acceptable). It takes no workspace.
  *
- * dir 0 solves Algorithm 3 (comp = fc, xfer = pt), dir 1 Algorithm 4
- * (comp = bc, xfer = gt); inputs, outputs and per-instance status are exactly
- * those of dc_schedule_forward_batch / dc_schedule_backward_batch.
+ * dir 0 is the forward call's problem (comp = fc, xfer = pt), dir 1 the
+ * backward call's (comp = bc, xfer = gt); inputs, outputs and per-instance
+ * status are exactly those of dc_schedule_forward_batch /
+ * dc_schedule_backward_batch, including a NULL status (a failed instance's
+ * makespan then carries -status).
  * Limits: 1 <= L <= 16 (else DC_ERR_BAD_SHAPE); batch <= 1,048,576
  * (DC_STATIC_MAX_BATCH; a larger batch returns DC_ERR_WORKSPACE, launching
  * nothing).
@@ -226,9 +228,11 @@ dc_status dc_eval_timeline_batch(int64_t batch, int32_t L, int32_t dir, const in
  * GPU that loads the library until the process exits, shared by all calls on a
  * device: calls that overlap on one GPU race on it, so serialise them (one
  * stream, or an event between them). Each call clears what must start at zero.
- * The first call on a device looks up the array's device address (a
- * cudaGetSymbolAddress with that device current); make that first call before
- * any stream capture. No cudaMalloc, cudaFree or other allocating call is made.
+ * Every call looks up the array's device address on the current device
+ * (cudaGetSymbolAddress, which allocates nothing); on a device's first call
+ * that lookup also loads the library's device code there if needed, so make
+ * the first call on each device before any stream capture. No cudaMalloc,
+ * cudaFree or other allocating call is made.
  * ---------------------------------------------------------------------- */
 #define DC_STATIC_MAX_BATCH 1048576
 dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_t L, const int64_t *comp,

@@ -14,8 +14,6 @@
 // device shares it: calls that overlap on one GPU race on it and must be
 // serialised by the caller (one stream, or an event between them). The counter
 // that must start at zero is cleared on the caller's stream by each call.
-#include <mutex>
-
 #include "common.cuh"
 
 namespace dc {
@@ -26,26 +24,18 @@ constexpr size_t kStaticScratchBytes = 256 + size_t(kStaticMaxBatch) * 4;  // he
 
 __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-// In host code `g_static_scratch` names a host-side stand-in, not device memory:
-// the device address is looked up once per device, with that device current.
-constexpr int kMaxDevices = 64;
-void *g_static_addr[kMaxDevices] = {};
-std::mutex g_static_mutex;
-
+// In host code `g_static_scratch` names a host-side stand-in, not device memory.
+// Its device address on the current device is looked up on every call: the
+// lookup allocates nothing, and no address is kept that a re-created context
+// (after a cudaDeviceReset, say) could have moved. On the first call on a
+// device, the lookup also loads this library's device code there if that has
+// not happened yet, which is why that first call belongs before any capture.
 cudaError_t static_scratch(void **out)
 {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lock(g_static_mutex);
-    if (g_static_addr[dev] == nullptr) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_scratch);
-        if (e != cudaSuccess) return e;
-        g_static_addr[dev] = p;
-    }
-    *out = g_static_addr[dev];
+    *out = p;
     return cudaSuccess;
 }
 

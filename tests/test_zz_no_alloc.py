@@ -64,6 +64,35 @@ def test_static_scratch_matches_workspace_entry(dc, name, batch):
             assert ref["status"][11] == dc.DC_OK
 
 
+def test_static_scratch_null_status_and_nseg(dc):
+    """With nseg and status NULL, a failed instance reports -status in its
+    makespan; every other output equals the workspace entry's, on two calls in a
+    row through the shared scratch."""
+    import torch
+    cfg = wl.with_batch(wl.config("vgg16"), 50_000)
+    prof = dc.profile_gen(cfg)
+    B, L, W = cfg["batch"], cfg["L"], dc.words(cfg["L"])
+    prof["pt"][7, 0] = 1 << 34   # 64-bit instance: the work list is used
+    prof["fc"][13, 1] = -1       # negative cost
+    prof["dt"][21] = 1 << 51     # L * dt beyond 2^52
+    for d, (c, x) in ((dc.FWD, ("fc", "pt")), (dc.BWD, ("bc", "gt"))):
+        ref = dc.schedule(d, prof[c], prof[x], prof["dt"])
+        torch.cuda.synchronize()
+        ref = {k: v.cpu().numpy() for k, v in ref.items()}
+        for call in range(2):
+            out = _outputs(torch, B, W)
+            st = dc.dc_schedule_batch_static(d, B, L, prof[c], prof[x], prof["dt"],
+                                             out["makespan"], out["bits"], None, None)
+            assert st == dc.DC_OK, dc.dc_status_string(st)
+            torch.cuda.synchronize()
+            got = out["makespan"].cpu().numpy()
+            assert np.array_equal(got, ref["makespan"]), (d, call)
+            assert np.array_equal(out["bits"].cpu().numpy()[:, :W], ref["bits"][:, :W])
+            if d == dc.FWD:
+                assert got[13] == -dc.DC_ERR_NEGATIVE
+            assert got[21] == -dc.DC_ERR_RANGE
+
+
 def test_static_scratch_limits(dc):
     import torch
     big = dc.DC_STATIC_MAX_BATCH + 1
