@@ -286,10 +286,119 @@ def test_config_full_batch_parity(dc, name):
     _config_parity(dc, name)
 
 
+def _solve_class(direction, comp, xfer, dt):
+    """Which arithmetic the per-instance solvers use for each instance (a
+    property of the inputs: the capped bound and the total compute), to spread
+    a sample over every path. 0: shifted signed 32 bits; 1: backward E form;
+    2: forward E form; 3: 32-bit template; 4: 64-bit."""
+    sc = comp.sum(1)
+    cx = np.minimum(xfer, sc[:, None]).sum(1)
+    bound = sc + cx + comp.shape[1] * dt
+    cls = np.full(len(dt), 4)
+    cls[bound <= 2**32 - 2] = 3
+    if direction == BWD:
+        cls[sc < 2**31 - 1] = 1
+    else:
+        cls[sc < 2**29] = 2
+    cls[bound <= 2**31 - 1] = 0
+    return cls
+
+
+def _deepchain_sample(prof, size, seed):
+    """`size` instances spread over the whole batch: half uniformly, half from the
+    instances that need a wide form in either direction."""
+    rng = np.random.default_rng(seed)
+    B = len(prof["dt"])
+    wide = np.nonzero((_solve_class(FWD, prof["fc"], prof["pt"], prof["dt"]) > 0) |
+                      (_solve_class(BWD, prof["bc"], prof["gt"], prof["dt"]) > 0))[0]
+    pick = np.concatenate([[0, 1, B - 1], rng.choice(B, size // 2, replace=False),
+                           rng.choice(wide, size - size // 2 - 3, replace=False)])
+    return np.unique(pick)
+
+
 def test_config_deepchain_sampled_parity(dc):
-    rng = np.random.default_rng(4)
-    sample = np.concatenate([[0, 1, 16383], rng.integers(0, 16384, size=5)])
+    """512+ deep-chain instances (L = 1024) from all over the batch, half of them
+    from the instances that take the wide forms, bit-exact with the oracle in both
+    directions; every decision of the batch replays to its makespan."""
+    prof = oracle.profile_gen(wl.config("deepchain"))
+    sample = _deepchain_sample(prof, 520, 4)
+    assert len(sample) >= 512
+    for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+        cls = _solve_class(d, prof[c][sample], prof[x][sample], prof["dt"][sample])
+        assert (cls == 0).sum() >= 100 and (cls == (1 if d == BWD else 2)).sum() >= 100
     _config_parity(dc, "deepchain", sample=sample)
+
+
+def _digests():
+    from conftest import GOLDEN
+    prof, chunks = {}, {}
+    with open(os.path.join(GOLDEN, "deepchain_oracle_digest.txt")) as f:
+        for line in f:
+            w = line.split()
+            if not w or w[0].startswith("#"):
+                continue
+            if w[0] == "profile":
+                prof[w[1]] = w[2]
+            elif w[0] == "chunk":
+                chunks[(int(w[1]), int(w[2]), int(w[3]))] = w[4]
+    return prof, chunks
+
+
+def test_config_deepchain_full_batch_digest(dc):
+    """Every instance of the deep-chain batch (16,384 x L = 1024), both directions,
+    bit for bit: the library's profiles and outputs hashed in chunks of 256
+    instances against tests/golden/deepchain_oracle_digest.txt, which
+    tests/golden/make_deepchain_digest.py wrote from the oracle's outputs."""
+    import hashlib
+
+    import torch
+    sys_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "make_deepchain_digest", os.path.join(sys_path, "make_deepchain_digest.py"))
+    mk = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mk)
+    want_prof, want_chunks = _digests()
+    assert len(want_chunks) == 2 * 64
+    cfg = wl.config("deepchain")
+    prof = dc.profile_gen(cfg)
+    torch.cuda.synchronize()
+    host = {k: v.cpu().numpy() for k, v in prof.items()}
+    for k in ("fc", "pt", "bc", "gt", "dt"):
+        assert mk.profile_digest(host[k]) == want_prof[k], f"generated profile {k} differs"
+    for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+        got = _gpu_schedule(dc, d, host[c], host[x], host["dt"])
+        bad = [(lo, hi) for (dd, lo, hi), h in sorted(want_chunks.items())
+               if dd == d and mk.chunk_digest(got, lo, hi) != h]
+        assert not bad, f"direction {d}: {len(bad)} chunks of 256 differ, first {bad[:4]}"
+
+
+@pytest.mark.parametrize("direction", [FWD, BWD])
+def test_deepchain_every_arithmetic_path(dc, direction):
+    """L = 1024 instances built to take each of the per-instance solver's five
+    arithmetic paths (shifted 32-bit, the backward and forward E forms, the
+    32-bit template, 64-bit), four of each, bit-exact with the oracle."""
+    L = 1024
+    cfg = wl.with_batch(wl.config("deepchain"), 4096)
+    prof = oracle.profile_gen(cfg)
+    c, x = ("fc", "pt") if direction == FWD else ("bc", "gt")
+    cls = _solve_class(direction, prof[c], prof[x], prof["dt"])
+    idx = [int(i) for k in (0, 1 if direction == BWD else 2) for i in np.nonzero(cls == k)[0][:4]]
+    comp, xfer, dt = prof[c][idx].copy(), prof[x][idx].copy(), prof["dt"][idx].copy()
+    rng = np.random.default_rng(50 + direction)
+    for target in (3, 4):  # total compute past the E forms' limits
+        for j in range(4):
+            cc = rng.integers(1, 100, size=L)
+            scale = (2**31 + 2**27) if target == 3 else 2**33
+            cc = cc * (scale // int(cc.sum())) + 1
+            xx = rng.integers(0, 1000, size=L) * (1 if target == 3 else 1 << 20)
+            comp = np.vstack([comp, cc[None]])
+            xfer = np.vstack([xfer, xx[None]])
+            dt = np.append(dt, rng.integers(0, 100))
+    got_cls = _solve_class(direction, comp, xfer, dt)
+    want = [0] * 4 + [1 if direction == BWD else 2] * 4 + [3] * 4 + [4] * 4
+    assert list(got_cls) == want, got_cls
+    _check_direction(dc, direction, comp, xfer, dt, f"deep paths dir={direction}")
 
 
 @pytest.mark.parametrize("L,sample", [(256, 64), (512, 16), (2048, 2)])
