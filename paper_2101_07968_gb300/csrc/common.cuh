@@ -43,17 +43,27 @@ inline int64_t table_slots(int L)
 }
 
 size_t mid_scratch_bytes(int64_t batch, int L);  // dp_mid.cu
+size_t deep_slot_bytes(int L);                   // dp_deep.cu
+int64_t deep_slots_bound(int L);                 // dp_deep.cu
+
+// CTA-per-instance tables for the instances the deep-chain kernel lists (L >
+// kMidLMax): a few, within ~1 GiB.
+inline int64_t list_table_slots(int L)
+{
+    const int64_t per = tri_cells(L) * 8;
+    int64_t s = (int64_t(1) << 30) / per;
+    if (s > 152 * 4) s = 152 * 4;
+    if (s < 4) s = 4;
+    return s;
+}
 
 struct Workspace {
-    // Layout: [0, 256) header (work-list counter, tile ticket), [256, 256 + 4*batch)
-    // work list (L <= kMidLMax), then, 256-aligned, the looped kernel's traceback
-    // slots (17 <= L <= kMidLMax), then, 256-aligned, the per-CTA DP tables of the
-    // group kernel (L > kSmemTableLMax: the looped kernel's work list or, above
-    // kMidLMax, the whole batch).
-    static size_t list_bytes(int64_t batch, int L)
-    {
-        return L <= kMidLMax ? size_t(batch) * 4 : 0;
-    }
+    // Layout: [0, 256) header (work-list counter, tile ticket / instance ticket),
+    // [256, 256 + 4*batch) work list, then, 256-aligned, the looped kernel's
+    // traceback slots (17 <= L <= kMidLMax) or the deep-chain kernel's per-CTA
+    // slots (L > kMidLMax), then, 256-aligned, the per-CTA DP tables of the group
+    // kernel for the listed instances (L > kSmemTableLMax).
+    static size_t list_bytes(int64_t batch, int) { return size_t(batch) * 4; }
     static size_t table_offset(int64_t batch, int L)
     {
         return (256 + list_bytes(batch, L) + 255) / 256 * 256;
@@ -61,13 +71,21 @@ struct Workspace {
     static size_t slots(int64_t batch, int L)
     {
         if (L <= kSmemTableLMax) return 0;
-        int64_t s = table_slots(L);
+        const int64_t s = L > kMidLMax ? list_table_slots(L) : table_slots(L);
         return size_t(batch < s ? batch : s);
+    }
+    static int64_t deep_slots(int64_t batch, int L)
+    {
+        if (L <= kMidLMax) return 0;
+        const int64_t s = deep_slots_bound(L);
+        return batch < s ? batch : s;
     }
     static size_t group_tables_offset(int64_t batch, int L)
     {
         if (L > kSmallLMax && L <= kMidLMax)
             return (table_offset(batch, L) + mid_scratch_bytes(batch, L) + 255) / 256 * 256;
+        if (L > kMidLMax)
+            return table_offset(batch, L) + size_t(deep_slots(batch, L)) * deep_slot_bytes(L);
         return table_offset(batch, L);
     }
     static size_t bytes(int64_t batch, int L)
@@ -152,6 +170,11 @@ cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
                        uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream);
+cudaError_t launch_deep(bool forward, int64_t lo, int64_t count, int L, const int64_t *comp,
+                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
+                        uint32_t *list_count, uint32_t *list, void *slots, int64_t nslots,
+                        cudaStream_t stream);
 cudaError_t launch_eval(bool forward, int64_t batch, int L, const int64_t *comp,
                         const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                         int64_t *makespan, cudaStream_t stream);

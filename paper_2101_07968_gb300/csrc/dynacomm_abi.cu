@@ -46,10 +46,20 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
                             count, list, ws + Workspace::group_tables_offset(batch, L),
                             int64_t(Workspace::slots(batch, L)), stream);
     }
-    const int64_t slots = int64_t(Workspace::slots(batch, L));
-    return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                        nullptr, nullptr, ws + Workspace::group_tables_offset(batch, L), slots,
-                        stream);
+    // warp-per-instance pass over the batch (three shifted 32-bit forms), then
+    // the CTA-per-instance kernel over the instances it listed
+    uint32_t *count = reinterpret_cast<uint32_t *>(ws);
+    uint32_t *ticket = count + 1;
+    uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
+    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(uint32_t), stream);
+    if (e != cudaSuccess) return e;
+    e = launch_deep(forward, 0, batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket,
+                    count, list, ws + Workspace::table_offset(batch, L),
+                    Workspace::deep_slots(batch, L), stream);
+    if (e != cudaSuccess) return e;
+    return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, count,
+                        list, ws + Workspace::group_tables_offset(batch, L),
+                        int64_t(Workspace::slots(batch, L)), stream);
 }
 
 namespace {

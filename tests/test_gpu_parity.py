@@ -79,6 +79,20 @@ def test_dp_random_parity(dc, L, kind):
         _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
 
 
+@pytest.mark.parametrize("L", [257, 258, 300, 333, 512, 600])
+@pytest.mark.parametrize("kind", ["tie", "uni", "skew"])
+def test_dp_deep_random_parity(dc, L, kind):
+    """The warp-per-instance deep-chain kernel (L > 256) and its work list:
+    several waves of instances, odd and even L (odd L stages rows with plain
+    loads), tie-heavy inputs for the traceback's lowest-k rule."""
+    B = 45
+    gen = {"tie": wl.tie_heavy_instances, "uni": wl.random_instances,
+           "skew": wl.skewed_instances}[kind]
+    comp, xfer, dt = gen(3000 * L + len(kind), B, L)
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
+
+
 @pytest.mark.parametrize("L", [1, 2, 8, 16, 17, 54, 70, 100, 200])
 def test_dp_wide_values_parity(dc, L):
     """Instances whose bound exceeds 2^32 need 64-bit arithmetic; mix them with
