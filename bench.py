@@ -635,10 +635,10 @@ def run_ours(args):
         traffic = tr.get("bytes_per_launch")
     hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
     dp_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
-    # kernels of this library per step: the generator; per direction the 32-bit
-    # pass and the pass over its work list (L <= 256) or the per-instance kernel
-    # alone (L > 256); the two timeline replays
-    launches_per_step = 1 + 2 * (2 if L <= 256 else 1) + 2
+    # kernels of this library per step: the generator; per direction the first
+    # pass (split into several launches for long deep-chain batches) and the
+    # pass over its work list; the two timeline replays
+    launches_per_step = 1 + 2 * dc.dc_schedule_kernel_launches(B, L) + 2
     # both roofs of the DP pass; the one it comes closer to (the larger minimal
     # time at peak) binds and is reported, the other rides along
     alu_roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "Gtransitions/s",

@@ -111,11 +111,26 @@ dc_status dc_profile_gen(const dc_profile_cfg *cfg, int64_t *fc, int64_t *pt, in
 
 /* ------------------------------------------------------------------------
  * dc_schedule_workspace_bytes -- device scratch a schedule call needs for
- * (batch, L): a work list for instances whose values need 64-bit arithmetic
- * (L <= 256), traceback slots of the thread-per-instance kernel (17 <= L <= 256)
- * and, for L > 64, per-CTA DP tables. Pure host function, no CUDA call.
+ * (batch, L): a work list for instances that the first pass leaves to a
+ * second (values beyond its 32-bit forms, or an optimum with more segments
+ * than it keeps traceback columns for); traceback slots of the
+ * thread-per-instance kernel (17 <= L <= 256) or, for L > 256, the per-CTA
+ * slots of the warp-per-instance kernel with their flags and per-launch
+ * counters; for L > 64, per-CTA DP tables of the second pass. Pure host
+ * function, no CUDA call.
  * ---------------------------------------------------------------------- */
 size_t dc_schedule_workspace_bytes(int64_t batch, int32_t L);
+
+/* ------------------------------------------------------------------------
+ * dc_schedule_kernel_launches -- how many kernels one dc_schedule_forward_batch
+ * or dc_schedule_backward_batch call with (batch, L) launches: a first pass and
+ * a second pass over its work list; for L > 256 the first pass is split into
+ * launches of about 90 ms of work each (at least two resident waves), chained
+ * so that each may start while the one before drains. For counting only (the
+ * calls need no caller action per launch). Returns 0 for batch <= 0 or L out of
+ * range. Pure host function, no CUDA call.
+ * ---------------------------------------------------------------------- */
+int32_t dc_schedule_kernel_launches(int64_t batch, int32_t L);
 
 /* ------------------------------------------------------------------------
  * dc_schedule_forward_batch -- Algorithm 3 / Eq. 8 for every instance:

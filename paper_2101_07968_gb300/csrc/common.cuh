@@ -58,11 +58,12 @@ inline int64_t list_table_slots(int L)
 }
 
 struct Workspace {
-    // Layout: [0, 256) header (work-list counter, tile ticket / instance ticket),
-    // [256, 256 + 4*batch) work list, then, 256-aligned, the looped kernel's
-    // traceback slots (17 <= L <= kMidLMax) or the deep-chain kernel's per-CTA
-    // slots (L > kMidLMax), then, 256-aligned, the per-CTA DP tables of the group
-    // kernel for the listed instances (L > kSmemTableLMax).
+    // Layout: [0, 256) header (work-list counter, tile ticket), [256, 256 +
+    // 4*batch) work list, then, 256-aligned, the looped kernel's traceback slots
+    // (17 <= L <= kMidLMax) or, for L > kMidLMax, the deep-chain kernel's slot
+    // flags and per-launch tickets (4 bytes each) and, 256-aligned, its per-CTA
+    // slots; then, 256-aligned, the per-CTA DP tables of the group kernel for
+    // the listed instances (L > kSmemTableLMax).
     static size_t list_bytes(int64_t batch, int) { return size_t(batch) * 4; }
     static size_t table_offset(int64_t batch, int L)
     {
@@ -80,12 +81,16 @@ struct Workspace {
         const int64_t s = deep_slots_bound(L);
         return batch < s ? batch : s;
     }
+    static size_t deep_slots_offset(int64_t batch, int L)
+    {
+        return (table_offset(batch, L) + size_t(deep_slots(batch, L) + batch) * 4 + 255) / 256 * 256;
+    }
     static size_t group_tables_offset(int64_t batch, int L)
     {
         if (L > kSmallLMax && L <= kMidLMax)
             return (table_offset(batch, L) + mid_scratch_bytes(batch, L) + 255) / 256 * 256;
         if (L > kMidLMax)
-            return table_offset(batch, L) + size_t(deep_slots(batch, L)) * deep_slot_bytes(L);
+            return deep_slots_offset(batch, L) + size_t(deep_slots(batch, L)) * deep_slot_bytes(L);
         return table_offset(batch, L);
     }
     static size_t bytes(int64_t batch, int L)
@@ -170,11 +175,12 @@ cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
                        uint32_t *list_count, uint32_t *list, uint32_t *tb, cudaStream_t stream);
-cudaError_t launch_deep(bool forward, int64_t lo, int64_t count, int L, const int64_t *comp,
+cudaError_t launch_deep(bool forward, int64_t batch, int L, const int64_t *comp,
                         const int64_t *xfer, const int64_t *dt, int64_t *makespan,
-                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
-                        uint32_t *list_count, uint32_t *list, void *slots, int64_t nslots,
-                        cudaStream_t stream);
+                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *tickets,
+                        uint32_t *busy, uint32_t *list_count, uint32_t *list, void *slots,
+                        int64_t nslots, cudaStream_t stream);
+int64_t deep_launches(int64_t batch, int L);  // launches of one deep-chain pass (dp_deep.cu)
 cudaError_t launch_eval(bool forward, int64_t batch, int L, const int64_t *comp,
                         const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                         int64_t *makespan, cudaStream_t stream);

@@ -73,7 +73,7 @@ __host__ __device__ inline int deep_plan_max(int L) { return L / 32 + 2; }
 __host__ __device__ inline size_t deep_urow_off(int L) { return 16 + 2 * deep_pair_bytes(L); }
 __host__ __device__ inline size_t deep_bits_off(int L) { return deep_urow_off(L) + al16(size_t(L + 1) * 4); }
 __host__ __device__ inline size_t deep_plan_off(int L) { return deep_bits_off(L) + al16(size_t(words_for(L) + 1) * 4); }
-__host__ __device__ inline size_t deep_smem(int L) { return deep_plan_off(L) + size_t(deep_plan_max(L)) * 16 + 16; }
+__host__ __device__ inline size_t deep_smem(int L, int NW) { return deep_plan_off(L) + size_t(NW) * (deep_plan_max(L) + 1) * 16; }
 
 __host__ __device__ inline int64_t kept_cols(int L) { return L < kKeep ? L : kKeep; }
 __host__ __device__ inline int64_t kept_cells(int L)
@@ -100,8 +100,10 @@ struct DeepArgs {
     int32_t *nseg, *status;
     uint32_t *ticket;                // instances taken so far (zero before the launch)
     uint32_t *list_count, *list;     // instances left to the CTA-per-instance kernel
+    uint32_t *busy;                  // slot bitmap: bit set while a CTA holds the slot (zero before the first launch)
     unsigned char *slots;
     size_t slot_bytes;
+    int nslots;
     int bulk;                        // profile rows may be staged with cp.async.bulk
 };
 
@@ -164,11 +166,14 @@ __device__ __forceinline__ uint64_t warp_excl_scan_u64(uint64_t v, int lane)
 }
 __device__ __forceinline__ int32_t yclamp64(int64_t v) { return v < int64_t(kYCl) ? int32_t(v) : kYCl; }
 
-// One block of R strips (rows bot + l + 32 j, j < R, top = bot + 32 R - 1) of
-// column n: candidate loops, then the finalised rows written to the next
-// column's pairs, the kept table and the last row.
-template <int R, int FORM, bool FWD>
-__device__ __forceinline__ void block(int L, int n, int bot, int k_lo, bool far, int32_t gfar,
+// One block of R strips of column n: strip j holds rows b0 + S j + lane (S =
+// 32 x the warps sharing the instance; top = b0 + S (R-1) + 31). Candidates:
+// the rectangle k in [k_lo, b0 - 1] that every strip takes, then for each strip
+// J its own 32 k (strips above take them all, strip J the k below its row) and,
+// when S > 32, the gap up to the next strip (strips above J only). Then the
+// finalised rows go to the next column's pairs, the kept table and the last row.
+template <int R, int FORM, bool FWD, int S>
+__device__ __forceinline__ void block(int L, int n, int b0, int k_lo, bool far, int32_t gfar,
                                       int64_t dt, const int2 *__restrict__ cur, int2 *__restrict__ nxt,
                                       const int32_t *__restrict__ urow, int32_t *__restrict__ kept,
                                       int32_t *__restrict__ last, int koff, int lane)
@@ -177,12 +182,12 @@ __device__ __forceinline__ void block(int L, int n, int bot, int k_lo, bool far,
     const int32_t ndt1 = (FORM == kS32 && !FWD) ? int32_t(int64_t(n - 1) * dt) : 0;
 #pragma unroll
     for (int j = 0; j < R; ++j) {
-        int m = bot + lane + 32 * j;
+        int m = b0 + lane + S * j;
         m = m < 0 ? 0 : m;
         u[j] = urow[m] - ndt1;
         acc[j] = far ? gfar : kInf;
     }
-    // rectangle: k in [k_lo, bot - 1], every row
+    // rectangle: k in [k_lo, b0 - 1], every row
     int k = k_lo;
     if ((k + koff) & 1) {
         if (FORM == kEfwd) {  // k_lo - 1 may be a far k: take k_lo on its own
@@ -194,18 +199,21 @@ __device__ __forceinline__ void block(int L, int n, int bot, int k_lo, bool far,
             --k;  // k_lo - 1 = n - 2 is a neutral entry
         }
     }
-    const int4 *pp = reinterpret_cast<const int4 *>(cur + koff + k);
-    const int4 *pe = reinterpret_cast<const int4 *>(cur + koff + bot);
+    {
+        const int4 *pp = reinterpret_cast<const int4 *>(cur + koff + k);
+        const int4 *pe = reinterpret_cast<const int4 *>(cur + koff + b0);
 #pragma unroll 2
-    for (; pp < pe; ++pp) {
-        const int4 p = *pp;
+        for (; pp < pe; ++pp) {
+            const int4 p = *pp;
 #pragma unroll
-        for (int j = 0; j < R; ++j) acc[j] = __vimin3_s32(acc[j], va(u[j], p.x, p.y), va(u[j], p.z, p.w));
+            for (int j = 0; j < R; ++j)
+                acc[j] = __vimin3_s32(acc[j], va(u[j], p.x, p.y), va(u[j], p.z, p.w));
+        }
     }
-    // triangle: strip q's k range; strips above take every k, strip q k < its row
 #pragma unroll
     for (int q = 0; q < R; ++q) {
-        const int4 *tq = reinterpret_cast<const int4 *>(cur + koff + bot + 32 * q);
+        // strip q's own k: strips above take every k, strip q the k below its row
+        const int4 *tq = reinterpret_cast<const int4 *>(cur + koff + b0 + S * q);
 #pragma unroll 2
         for (int c = 0; c < 32; c += 2) {
             const int4 p = tq[c >> 1];
@@ -216,11 +224,22 @@ __device__ __forceinline__ void block(int L, int n, int bot, int k_lo, bool far,
             const int32_t c1 = c + 1 < lane ? va(u[q], p.z, p.w) : kInf;
             acc[q] = __vimin3_s32(acc[q], c0, c1);
         }
+        if (S > 32 && q + 1 < R) {  // the other warps' strips between q and q + 1
+            const int4 *pp = tq + 16;
+            const int4 *pe = tq + S / 2;
+#pragma unroll 2
+            for (; pp < pe; ++pp) {
+                const int4 p = *pp;
+#pragma unroll
+                for (int j = q + 1; j < R; ++j)
+                    acc[j] = __vimin3_s32(acc[j], va(u[j], p.x, p.y), va(u[j], p.z, p.w));
+            }
+        }
     }
     // finalise
 #pragma unroll
     for (int j = 0; j < R; ++j) {
-        const int m = bot + lane + 32 * j;
+        const int m = b0 + lane + S * j;
         if (m < n) continue;
         const int2 c = cur[m + koff];
         int32_t X, nx, ny;
@@ -244,16 +263,16 @@ __device__ __forceinline__ void block(int L, int n, int bot, int k_lo, bool far,
     }
 }
 
-template <int FORM, bool FWD>
-__device__ __forceinline__ void run_block(int R, int L, int n, int bot, int k_lo, bool far,
+template <int FORM, bool FWD, int S>
+__device__ __forceinline__ void run_block(int R, int L, int n, int b0, int k_lo, bool far,
                                           int32_t gfar, int64_t dt, const int2 *cur, int2 *nxt,
                                           const int32_t *urow, int32_t *kept, int32_t *last,
                                           int koff, int lane)
 {
-#define DC_DEEP_BLOCK(RR)                                                                         \
-    case RR:                                                                                      \
-        block<RR, FORM, FWD>(L, n, bot, k_lo, far, gfar, dt, cur, nxt, urow, kept, last, koff, \
-                             lane);                                                               \
+#define DC_DEEP_BLOCK(RR)                                                                        \
+    case RR:                                                                                     \
+        block<RR, FORM, FWD, S>(L, n, b0, k_lo, far, gfar, dt, cur, nxt, urow, kept, last, koff, \
+                                lane);                                                           \
         break;
     switch (R) {
         DC_DEEP_BLOCK(1) DC_DEEP_BLOCK(2) DC_DEEP_BLOCK(3) DC_DEEP_BLOCK(4)
@@ -263,11 +282,23 @@ __device__ __forceinline__ void run_block(int R, int L, int n, int bot, int k_lo
 #undef DC_DEEP_BLOCK
 }
 
-// The column loop of one form: columns 2..L, blocks from the plan.
-template <int FORM, bool FWD>
-__device__ void fill(int L, int64_t dt, int2 *XY0, int2 *XY1, const int32_t *urow,
-                     const int4 *plan, int nplan, int32_t *kept, int32_t *last, int koff, int lane)
+template <int NW>
+__device__ __forceinline__ void cta_sync()
 {
+    if (NW == 1)
+        __syncwarp();
+    else
+        __syncthreads();
+}
+
+// The column loop of one form: columns 2..L, each warp its plan's blocks, one
+// CTA barrier per column (the next column reads every warp's rows).
+template <int FORM, bool FWD, int NW>
+__device__ void fill(int L, int64_t dt, int2 *XY0, int2 *XY1, const int32_t *urow,
+                     const int4 *plan, int nplan, int32_t *kept, int32_t *last, int koff, int tid)
+{
+    constexpr int S = 32 * NW;
+    const int lane = tid & 31;
     for (int n = 2; n <= L; ++n) {
         const int2 *cur = (n - 1) & 1 ? XY1 : XY0;
         int2 *nxt = n & 1 ? XY1 : XY0;
@@ -275,9 +306,9 @@ __device__ void fill(int L, int64_t dt, int2 *XY0, int2 *XY1, const int32_t *uro
             const int4 b = plan[e];  // top, strips, kF
             const int top = b.x;
             if (top < n) break;
-            const int bot0 = top - 32 * b.y + 1;
-            const int jmin = n > bot0 ? (n - bot0) >> 5 : 0;
-            const int bot = bot0 + 32 * jmin;
+            const int b00 = top - 31 - S * (b.y - 1);
+            const int jmin = n - b00 - 31 > 0 ? (n - b00 - 31 + S - 1) / S : 0;
+            const int b0 = b00 + S * jmin;
             int k_lo = n - 1;
             bool far = false;
             int32_t gfar = 0;
@@ -286,27 +317,64 @@ __device__ void fill(int L, int64_t dt, int2 *XY0, int2 *XY1, const int32_t *uro
                 gfar = cur[b.z - 1 + koff].y;  // G[kF - 1]
                 k_lo = b.z;
             }
-            run_block<FORM, FWD>(b.y - jmin, L, n, bot, k_lo, far, gfar, dt, cur, nxt, urow, kept,
-                                 last, koff, lane);
+            run_block<FORM, FWD, S>(b.y - jmin, L, n, b0, k_lo, far, gfar, dt, cur, nxt, urow,
+                                    kept, last, koff, lane);
         }
         // entries n-2 and n-1 of the new column's pairs are stale: neutral
-        if (lane < 2 && n - 2 + lane >= 0) nxt[n - 2 + lane + koff].y = kInf;
-        __syncwarp();
+        if (tid < 2 && n - 2 + tid >= 0) nxt[n - 2 + tid + koff].y = kInf;
+        cta_sync<NW>();
     }
 }
 
-template <bool FWD>
-__global__ void __launch_bounds__(32) deep_kernel(DeepArgs a)
+template <bool FWD, int NW>
+__global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(DeepArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    const int L = a.L, lane = threadIdx.x, W = words_for(L), koff = deep_koff(L);
+    constexpr int S = 32 * NW;
+    const int L = a.L, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int W = words_for(L), koff = deep_koff(L), PM = deep_plan_max(L);
     uint64_t *bar = reinterpret_cast<uint64_t *>(smem);
+    volatile int32_t *ctl = reinterpret_cast<volatile int32_t *>(smem + 8);  // instance, flag
     int2 *XY0 = reinterpret_cast<int2 *>(smem + 16);
     int2 *XY1 = reinterpret_cast<int2 *>(smem + 16 + deep_pair_bytes(L));
     int32_t *urow = reinterpret_cast<int32_t *>(smem + deep_urow_off(L));
     uint32_t *bitsw = reinterpret_cast<uint32_t *>(smem + deep_bits_off(L));
-    int4 *plan = reinterpret_cast<int4 *>(smem + deep_plan_off(L));
-    unsigned char *slot = a.slots + size_t(blockIdx.x) * a.slot_bytes;
+    int4 *plans = reinterpret_cast<int4 *>(smem + deep_plan_off(L));
+    int4 *plan = plans + warp * (PM + 1);
+
+    // The next launch of a split batch may start filling SMs as this one's CTAs
+    // exit (programmatic dependent launch); it shares no data with this one.
+    pdl_trigger();
+    // Claim a free slot: at most one resident wave of CTAs lives at a time, over
+    // this launch and the next, and there are at least that many slots. Each
+    // bitmap word is tried from a free bit until one is won or none is left.
+    if (tid == 0) {
+        int got = -1;
+        const int nw = (a.nslots + 31) / 32;
+        for (int p = 0; p < nw && got < 0; ++p) {
+            const int w = int((blockIdx.x / 32u + unsigned(p)) % unsigned(nw));
+            const int nbits = min(32, a.nslots - 32 * w);
+            const uint32_t full = nbits == 32 ? 0xffffffffu : ((1u << nbits) - 1u);
+            uint32_t v = *reinterpret_cast<volatile uint32_t *>(a.busy + w);
+            for (int tries = 0; tries < 32 && (v & full) != full; ++tries) {
+                const int b = __ffs(~v & full) - 1;
+                const uint32_t old = atomicOr(a.busy + w, 1u << b);
+                if (!(old & (1u << b))) {
+                    got = 32 * w + b;
+                    break;
+                }
+                v = old | (1u << b);
+            }
+        }
+        reinterpret_cast<volatile int32_t *>(smem + 8)[1] = got;
+    }
+    __syncthreads();
+    const int slot_id = reinterpret_cast<volatile int32_t *>(smem + 8)[1];
+    if (slot_id < 0) {  // every slot held (not expected): leave the instances to the other CTAs
+        pdl_wait();
+        return;
+    }
+    unsigned char *slot = a.slots + size_t(slot_id) * a.slot_bytes;
     uint64_t *P64 = reinterpret_cast<uint64_t *>(slot);
     int32_t *last = reinterpret_cast<int32_t *>(slot + slot_last_off(L));
     int32_t *Gk = reinterpret_cast<int32_t *>(slot + slot_g_off(L));
@@ -314,301 +382,321 @@ __global__ void __launch_bounds__(32) deep_kernel(DeepArgs a)
     uint64_t *rawc = reinterpret_cast<uint64_t *>(XY0);
     uint64_t *rawx = reinterpret_cast<uint64_t *>(XY1);
 
-    if (a.bulk && lane == 0) mbar_init(bar);
-    __syncwarp();
+    if (a.bulk && tid == 0) mbar_init(bar);
+    __syncthreads();
     uint32_t phase = 0;
     const int chunk = (L + 31) / 32;
     const int r_lo = 1 + lane * chunk, r_hi = min(L, r_lo + chunk - 1);
     auto col = [&](int r) { return FWD ? r - 1 : L - r; };
+    enum { kListed = -1, kAbort = -2 };
 
     for (;;) {
-        uint32_t jt = 0;
-        if (lane == 0) jt = atomicAdd(a.ticket, 1u);
-        jt = __shfl_sync(0xffffffffu, jt, 0);
+        if (tid == 0) ctl[0] = int32_t(atomicAdd(a.ticket, 1u));
+        __syncthreads();
+        const uint32_t jt = uint32_t(ctl[0]);
         if (int64_t(jt) >= a.count) break;
         const int64_t i = a.lo + int64_t(jt);
         const int64_t dti = a.dt[i];
+        uint64_t sx = 0, shift = 0;  // warp 0: raw transfer total, capped-off transfer
 
-        // ---- profile rows into shared memory
-        if (a.bulk) {
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) {
-                mbar_expect(bar, uint32_t(16) * uint32_t(L));
-                bulk_g2s(rawc, a.comp + i * L, uint32_t(8) * uint32_t(L), bar);
-                bulk_g2s(rawx, a.xfer + i * L, uint32_t(8) * uint32_t(L), bar);
-            }
-            const bool ok = mbar_wait(bar, phase, 1 << 22);
-            phase ^= 1u;
-            if (!__all_sync(0xffffffffu, ok)) {
-                // the copies did not land in time: wait once more before the
-                // buffers are given up, then leave the instance failed
-                const bool late = mbar_wait(bar, phase ^ 1u, 1 << 22);
+        // ---- warp 0: rows, checks, form, prefix sums, column 1
+        if (warp == 0) {
+            int flag = 0;
+            bool staged = true;
+            if (a.bulk) {
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
                 if (lane == 0) {
-                    a.makespan[i] = -int64_t(DC_ERR_INTERNAL);
-                    if (a.nseg) a.nseg[i] = 0;
-                    if (a.status) a.status[i] = DC_ERR_INTERNAL;
+                    mbar_expect(bar, uint32_t(16) * uint32_t(L));
+                    bulk_g2s(rawc, a.comp + i * L, uint32_t(8) * uint32_t(L), bar);
+                    bulk_g2s(rawx, a.xfer + i * L, uint32_t(8) * uint32_t(L), bar);
                 }
-                for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
-                if (!__all_sync(0xffffffffu, late)) return;  // buffers may still be written
-                continue;
-            }
-        } else {
-            for (int c = lane; c < L; c += 32) {
-                rawc[c] = uint64_t(__ldg(a.comp + i * L + c));
-                rawx[c] = uint64_t(__ldg(a.xfer + i * L + c));
-            }
-            __syncwarp();
-        }
-
-        // ---- checks and totals
-        bool neg = dti < 0, big = (dti >> 52) != 0;
-        uint64_t sc = 0, sx = 0;
-        for (int r = r_lo; r <= r_hi; ++r) {
-            const int64_t cv = int64_t(rawc[col(r)]), xv = int64_t(rawx[col(r)]);
-            neg |= (cv < 0) | (xv < 0);
-            big |= ((cv | xv) >> 52) != 0;
-            sc += uint64_t(cv);
-            sx += uint64_t(xv);
-        }
-        neg = __any_sync(0xffffffffu, neg);
-        big = __any_sync(0xffffffffu, big);
-        sc = warp_sum_u64(sc);
-        sx = warp_sum_u64(sx);
-        int st = DC_OK;
-        if (neg)
-            st = DC_ERR_NEGATIVE;
-        else if (big || exceeds_range(L, dti, sc, sx))
-            st = DC_ERR_RANGE;
-        if (st != DC_OK) {
-            if (lane == 0) {
-                a.makespan[i] = -int64_t(st);
-                if (a.nseg) a.nseg[i] = 0;
-                if (a.status) a.status[i] = st;
-            }
-            for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
-            __syncwarp();
-            continue;
-        }
-        // capped transfers; the arithmetic form
-        uint64_t cx = 0, cc = 0;
-        for (int r = r_lo; r <= r_hi; ++r) {
-            const uint64_t xv = rawx[col(r)];
-            cx += xv < sc ? xv : sc;
-            cc += rawc[col(r)];
-        }
-        const uint64_t cx_lane = cx, cc_lane = cc;
-        cx = warp_sum_u64(cx);
-        const uint64_t shift = sx - cx;
-        const uint64_t bound = sc + cx + uint64_t(L) * uint64_t(dti);
-        int form;
-        if (bound <= kShiftedLimit)
-            form = kS32;
-        else if (!FWD && sc < uint64_t(kYCl))
-            form = kEbwd;
-        else if (FWD && sc < (uint64_t(1) << 29))
-            form = kEfwd;
-        else
-            form = -1;
-        if (form < 0) {  // 32-bit or 64-bit literal template: the CTA-per-instance kernel
-            if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
-            __syncwarp();
-            continue;
-        }
-        // prefix sums in processing order: comp (below 2^31) into urow, capped
-        // transfers (64-bit) into the slot
-        {
-            uint64_t oc = warp_excl_scan_u64(cc_lane, lane), ox = warp_excl_scan_u64(cx_lane, lane);
-            // every lane reads its chunk before any lane's prefix lands in urow /
-            // the slot (they do not overlap the staged rows)
-            for (int r = r_lo; r <= r_hi; ++r) {
-                const uint64_t xv = rawx[col(r)];
-                oc += rawc[col(r)];
-                ox += xv < sc ? xv : sc;
-                urow[r] = int32_t(oc);
-                P64[r] = ox;
-            }
-            if (lane == 0) {
-                urow[0] = 0;
-                P64[0] = 0;
-            }
-            for (int w = lane; w < W + 1; w += 32) bitsw[w] = 0u;
-        }
-        __syncwarp();
-        // column 1 and the row terms
-        const int32_t fcL = urow[L];
-        __syncwarp();  // every lane has fcL before urow[L] is overwritten
-        for (int m = lane; m <= L; m += 32) {
-            const int32_t CF = urow[m];
-            const uint64_t P = P64[m];
-            int32_t u, x, y, X;
-            if (form == kS32) {
-                if (FWD) {
-                    u = int32_t(dti) + int32_t(P);
-                    x = fcL - CF;
-                    y = fcL + int32_t(P);
-                } else {
-                    u = CF;
-                    x = -int32_t(P);
-                    y = CF;
+                const bool ok = mbar_wait(bar, phase, 1 << 22);
+                phase ^= 1u;
+                if (!__all_sync(0xffffffffu, ok)) {
+                    // the copies did not land in time: wait once more before the
+                    // buffers are given up, then leave the instance failed
+                    const bool late = mbar_wait(bar, phase ^ 1u, 1 << 22);
+                    if (lane == 0) {
+                        a.makespan[i] = -int64_t(DC_ERR_INTERNAL);
+                        if (a.nseg) a.nseg[i] = 0;
+                        if (a.status) a.status[i] = DC_ERR_INTERNAL;
+                    }
+                    for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
+                    staged = false;
+                    flag = __all_sync(0xffffffffu, late) ? int(kListed) : int(kAbort);
                 }
-                X = y;
-            } else if (form == kEbwd) {
-                u = CF;
-                x = -yclamp64(dti + int64_t(P));
-                y = CF;
-                X = CF;
             } else {
-                u = int32_t(uint32_t(0) - uint32_t(dti) - uint32_t(P));
-                x = int32_t(uint32_t(fcL) + uint32_t(P));
-                y = fcL - CF;
-                Gk[m] = y;
-                X = CF;
+                for (int c = lane; c < L; c += 32) {
+                    rawc[c] = uint64_t(__ldg(a.comp + i * L + c));
+                    rawx[c] = uint64_t(__ldg(a.xfer + i * L + c));
+                }
+                __syncwarp();
             }
-            urow[m] = u;
-            XY1[m + koff] = make_int2(x, m == 0 ? kInf : y);
-            if (m >= 1) kept[tri_index(L, m, 1)] = X;
-            if (m == L) last[1] = X;
-        }
-        for (int e = lane; e < koff; e += 32) {
-            XY0[e] = make_int2(0, kInf);
-            XY1[e] = make_int2(0, kInf);
-        }
-        __syncwarp();
-
-        // ---- block plan (lane 0)
-        if (lane == 0) {
-            int np = 0, top = L;
-            bool ok = true;
-            while (top >= 1) {
-                if (form != kEfwd) {
-                    plan[np++] = make_int4(top, kMaxStrips, 0, 0);
-                    top -= 32 * kMaxStrips;
-                    continue;
+            if (staged) {
+                bool neg = dti < 0, big = (dti >> 52) != 0;
+                uint64_t sc = 0;
+                for (int r = r_lo; r <= r_hi; ++r) {
+                    const int64_t cv = int64_t(rawc[col(r)]), xv = int64_t(rawx[col(r)]);
+                    neg |= (cv < 0) | (xv < 0);
+                    big |= ((cv | xv) >> 52) != 0;
+                    sc += uint64_t(cv);
+                    sx += uint64_t(xv);
                 }
-                int R = kMaxStrips;
-                for (; R >= 1; R >>= 1) {
-                    const int botc = max(top - 32 * R + 1, 1);
-                    const int64_t span = int64_t(P64[top] - P64[botc]);
-                    if (span <= kSpanLimit && dti + span <= kTwo31) break;
-                }
-                if (R < 1) {
-                    ok = false;
-                    break;
-                }
-                // kF: first k with P[k] >= P[top] + dt - 2^31 (at most the block's bottom)
-                const int64_t thr = int64_t(P64[top]) + dti - kTwo31;
-                int lo = 0, hi = max(top - 32 * R + 1, 1);
-                while (lo < hi) {
-                    const int mid = (lo + hi) >> 1;
-                    if (int64_t(P64[mid]) < thr)
-                        lo = mid + 1;
+                neg = __any_sync(0xffffffffu, neg);
+                big = __any_sync(0xffffffffu, big);
+                sc = warp_sum_u64(sc);
+                sx = warp_sum_u64(sx);
+                int st = DC_OK;
+                if (neg)
+                    st = DC_ERR_NEGATIVE;
+                else if (big || exceeds_range(L, dti, sc, sx))
+                    st = DC_ERR_RANGE;
+                if (st != DC_OK) {
+                    if (lane == 0) {
+                        a.makespan[i] = -int64_t(st);
+                        if (a.nseg) a.nseg[i] = 0;
+                        if (a.status) a.status[i] = st;
+                    }
+                    for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
+                    flag = kListed;  // done: nothing for the other warps
+                } else {
+                    // capped transfers; the arithmetic form
+                    uint64_t cx = 0, cc = 0;
+                    for (int r = r_lo; r <= r_hi; ++r) {
+                        const uint64_t xv = rawx[col(r)];
+                        cx += xv < sc ? xv : sc;
+                        cc += rawc[col(r)];
+                    }
+                    const uint64_t cx_lane = cx, cc_lane = cc;
+                    cx = warp_sum_u64(cx);
+                    shift = sx - cx;
+                    const uint64_t bound = sc + cx + uint64_t(L) * uint64_t(dti);
+                    if (bound <= kShiftedLimit)
+                        flag = kS32;
+                    else if (!FWD && sc < uint64_t(kYCl))
+                        flag = kEbwd;
+                    else if (FWD && sc < (uint64_t(1) << 29))
+                        flag = kEfwd;
                     else
-                        hi = mid;
+                        flag = kListed;
+                    if (flag == kListed) {  // 32/64-bit literal template: the CTA-per-instance kernel
+                        if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+                    } else {
+                        // prefix sums in processing order: comp (below 2^31) into
+                        // urow, capped transfers (64-bit) into the slot
+                        uint64_t oc = warp_excl_scan_u64(cc_lane, lane);
+                        uint64_t ox = warp_excl_scan_u64(cx_lane, lane);
+                        for (int r = r_lo; r <= r_hi; ++r) {
+                            const uint64_t xv = rawx[col(r)];
+                            oc += rawc[col(r)];
+                            ox += xv < sc ? xv : sc;
+                            urow[r] = int32_t(oc);
+                            P64[r] = ox;
+                        }
+                        if (lane == 0) {
+                            urow[0] = 0;
+                            P64[0] = 0;
+                        }
+                        for (int w = lane; w < W + 1; w += 32) bitsw[w] = 0u;
+                        __syncwarp();
+                        // column 1 and the row terms
+                        const int32_t fcL = urow[L];
+                        __syncwarp();  // every lane has fcL before urow[L] is overwritten
+                        for (int m = lane; m <= L; m += 32) {
+                            const int32_t CF = urow[m];
+                            const uint64_t P = P64[m];
+                            int32_t u, x, y, X;
+                            if (flag == kS32) {
+                                if (FWD) {
+                                    u = int32_t(dti) + int32_t(P);
+                                    x = fcL - CF;
+                                    y = fcL + int32_t(P);
+                                } else {
+                                    u = CF;
+                                    x = -int32_t(P);
+                                    y = CF;
+                                }
+                                X = y;
+                            } else if (flag == kEbwd) {
+                                u = CF;
+                                x = -yclamp64(dti + int64_t(P));
+                                y = CF;
+                                X = CF;
+                            } else {
+                                u = int32_t(uint32_t(0) - uint32_t(dti) - uint32_t(P));
+                                x = int32_t(uint32_t(fcL) + uint32_t(P));
+                                y = fcL - CF;
+                                Gk[m] = y;
+                                X = CF;
+                            }
+                            urow[m] = u;
+                            XY1[m + koff] = make_int2(x, m == 0 ? kInf : y);
+                            if (m >= 1) kept[tri_index(L, m, 1)] = X;
+                            if (m == L) last[1] = X;
+                        }
+                        for (int e = lane; e < koff; e += 32) {
+                            XY0[e] = make_int2(0, kInf);
+                            XY1[e] = make_int2(0, kInf);
+                        }
+                    }
                 }
-                plan[np++] = make_int4(top, R, lo, 0);
-                top -= 32 * R;
             }
-            plan[deep_plan_max(L)] = make_int4(ok ? np : -1, 0, 0, 0);
+            if (lane == 0) ctl[1] = flag;
         }
-        __syncwarp();
-        const int nplan = plan[deep_plan_max(L)].x;
-        if (nplan < 0) {  // blocks narrower than 32 rows: the CTA-per-instance kernel
-            if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
-            __syncwarp();
+        __syncthreads();
+        const int form = ctl[1];
+        if (form == kAbort) {  // the staging buffers may still be written: keep the slot
+            pdl_wait();
+            return;
+        }
+        if (form < 0) {
+            __syncthreads();  // ctl is read by every thread before the next ticket
             continue;
         }
+
+        // ---- each warp's block plan: its strips t = warp, warp + NW, ... from
+        // the top (strip t holds rows L - 32 t - 31 .. L - 32 t), up to 8 per block
+        if (lane == 0) {
+            const int T = (L + 31) / 32;
+            int np = 0, t = warp;
+            bool ok = true;
+            while (t < T) {
+                const int avail = (T - 1 - t) / NW + 1;
+                int R = avail < kMaxStrips ? avail : kMaxStrips;
+                const int top = L - 32 * t;
+                int kF = 0;
+                if (form == kEfwd) {
+                    for (; R >= 1; --R) {
+                        const int botc = max(top - 31 - S * (R - 1), 1);
+                        const int64_t span = int64_t(P64[top] - P64[botc]);
+                        if (span <= kSpanLimit && dti + span <= kTwo31) break;
+                    }
+                    if (R < 1) {
+                        ok = false;
+                        break;
+                    }
+                    // kF: first k with P[k] >= P[top] + dt - 2^31 (at most the block's bottom)
+                    const int64_t thr = int64_t(P64[top]) + dti - kTwo31;
+                    int lo = 0, hi = max(top - 31 - S * (R - 1), 1);
+                    while (lo < hi) {
+                        const int mid = (lo + hi) >> 1;
+                        if (int64_t(P64[mid]) < thr)
+                            lo = mid + 1;
+                        else
+                            hi = mid;
+                    }
+                    kF = lo;
+                }
+                plan[np++] = make_int4(top, R, kF, 0);
+                t += R * NW;
+            }
+            plan[PM] = make_int4(ok ? np : -1, 0, 0, 0);
+        }
+        __syncthreads();
+        bool planned = true;
+        for (int w = 0; w < NW; ++w) planned &= plans[w * (PM + 1) + PM].x >= 0;
+        if (!planned) {  // blocks narrower than one strip: the CTA-per-instance kernel
+            if (tid == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+            __syncthreads();
+            continue;
+        }
+        const int nplan = plan[PM].x;
 
         // ---- columns 2..L
         if (form == kS32)
-            fill<kS32, FWD>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, lane);
+            fill<kS32, FWD, NW>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, tid);
         else if (form == kEbwd)
-            fill<kEbwd, FWD>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, lane);
+            fill<kEbwd, FWD, NW>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, tid);
         else
-            fill<kEfwd, FWD>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, lane);
+            fill<kEfwd, FWD, NW>(L, dti, XY0, XY1, urow, plan, nplan, kept, last, koff, tid);
+        __syncthreads();
 
-        // ---- lowest n minimising the makespan
-        int64_t bv = INT64_MAX;
-        int bn = 0x7fffffff;
-        const int64_t toB = (form == kS32 && FWD) ? int64_t(dti) - int64_t(urow[L]) : 0;
-        for (int n = 1 + lane; n <= L; n += 32) {
-            const int64_t v = int64_t(last[n]) + toB + int64_t(n) * dti;
-            if (v < bv) {
-                bv = v;
-                bn = n;
+        // ---- warp 0: lowest n minimising the makespan, then the traceback
+        if (warp == 0) {
+            int64_t bv = INT64_MAX;
+            int bn = 0x7fffffff;
+            const int64_t toB = (form == kS32 && FWD) ? int64_t(dti) - int64_t(urow[L]) : 0;
+            for (int n = 1 + lane; n <= L; n += 32) {
+                const int64_t v = int64_t(last[n]) + toB + int64_t(n) * dti;
+                if (v < bv) {
+                    bv = v;
+                    bn = n;
+                }
             }
-        }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const int64_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int on = __shfl_xor_sync(0xffffffffu, bn, o);
-            if (ov < bv || (ov == bv && on < bn)) {
-                bv = ov;
-                bn = on;
+            for (int o = 16; o > 0; o >>= 1) {
+                const int64_t ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                const int on = __shfl_xor_sync(0xffffffffu, bn, o);
+                if (ov < bv || (ov == bv && on < bn)) {
+                    bv = ov;
+                    bn = on;
+                }
             }
-        }
-        const int s = bn;
-        if (s - 1 > kKeep) {  // the traceback needs columns beyond the kept ones
-            if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
-            __syncwarp();
-            continue;
-        }
-
-        // ---- traceback: Path[m][n] = the lowest k whose candidate equals the cell
-        int err = 0, m = L, n = s;
-        const int2 *V = XY1;  // S32: x = V[k] in every entry k >= 1 of the column-1 buffer
-        while (n > 1) {
-            const int32_t Xmn = (m == L && n == s) ? last[s] : kept[tri_index(L, m, n)];
-            const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
-            int found = -1;
-            for (int k0 = n - 1; k0 < m; k0 += 32) {
-                const int k = k0 + lane;
-                bool match = false;
-                if (k < m) {
-                    const int32_t Xk = kept[pbase + k];
-                    if (form == kS32) {
-                        const int32_t u = FWD ? urow[m] : urow[m] - int32_t(int64_t(n - 1) * dti);
-                        const int32_t target = FWD ? Xmn + int32_t(dti) : Xmn;
-                        match = va(u, V[k + koff].x, Xk) == target;
-                    } else if (form == kEbwd) {
-                        const int32_t y = yclamp64(int64_t(n - 1) * dti + int64_t(P64[k]));
-                        match = max(Xk, urow[m] - y) == Xmn;
-                    } else {
-                        const int64_t Q = dti + int64_t(P64[m]);
-                        const int64_t g = Gk[k];
-                        const int64_t x = int64_t(Xk) + g + int64_t(P64[k]) - Q;
-                        match = (x > g ? x : g) == int64_t(Xmn) + Gk[m];
+            const int s = bn;
+            if (s - 1 > kKeep) {  // the traceback needs columns beyond the kept ones
+                if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+            } else {
+                // Path[m][n] = the lowest k whose candidate equals the cell
+                int err = 0, m = L, n = s;
+                const int2 *V = XY1;  // S32: x = V[k] in every entry k >= 1 of the column-1 buffer
+                while (n > 1) {
+                    const int32_t Xmn = (m == L && n == s) ? last[s] : kept[tri_index(L, m, n)];
+                    const int64_t pbase = tri_col(L, n - 1) - (n - 1);  // + k gives (k, n-1)
+                    int found = -1;
+                    for (int k0 = n - 1; k0 < m; k0 += 32) {
+                        const int k = k0 + lane;
+                        bool match = false;
+                        if (k < m) {
+                            const int32_t Xk = kept[pbase + k];
+                            if (form == kS32) {
+                                const int32_t u = FWD ? urow[m] : urow[m] - int32_t(int64_t(n - 1) * dti);
+                                const int32_t target = FWD ? Xmn + int32_t(dti) : Xmn;
+                                match = va(u, V[k + koff].x, Xk) == target;
+                            } else if (form == kEbwd) {
+                                const int32_t y = yclamp64(int64_t(n - 1) * dti + int64_t(P64[k]));
+                                match = max(Xk, urow[m] - y) == Xmn;
+                            } else {
+                                const int64_t Q = dti + int64_t(P64[m]);
+                                const int64_t g = Gk[k];
+                                const int64_t x = int64_t(Xk) + g + int64_t(P64[k]) - Q;
+                                match = (x > g ? x : g) == int64_t(Xmn) + Gk[m];
+                            }
+                        }
+                        const unsigned bal = __ballot_sync(0xffffffffu, match);
+                        if (bal) {
+                            found = k0 + __ffs(bal) - 1;
+                            break;
+                        }
                     }
+                    if (found < 0) {
+                        err = 1;
+                        break;
+                    }
+                    if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
+                    __syncwarp();
+                    m = found;
+                    n -= 1;
                 }
-                const unsigned bal = __ballot_sync(0xffffffffu, match);
-                if (bal) {
-                    found = k0 + __ffs(bal) - 1;
-                    break;
+                __syncwarp();
+                if (lane == 0) {
+                    const uint64_t mk = form == kS32 ? uint64_t(bv) + sx : uint64_t(bv) + P64[L] + shift;
+                    a.makespan[i] = err ? -int64_t(DC_ERR_INTERNAL) : int64_t(mk);
+                    if (a.nseg) a.nseg[i] = err ? 0 : s;
+                    if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
                 }
+                for (int w = lane; w < W; w += 32) a.bits[i * W + w] = err ? 0u : bitsw[w];
             }
-            if (found < 0) {
-                err = 1;
-                break;
-            }
-            if (lane == 0) bitsw[(found - 1) >> 5] |= 1u << ((found - 1) & 31);
-            __syncwarp();
-            m = found;
-            n -= 1;
         }
-        __syncwarp();
-        if (lane == 0) {
-            uint64_t mk;
-            if (form == kS32)
-                mk = uint64_t(bv) + sx;
-            else
-                mk = uint64_t(bv) + P64[L] + shift;
-            a.makespan[i] = err ? -int64_t(DC_ERR_INTERNAL) : int64_t(mk);
-            if (a.nseg) a.nseg[i] = err ? 0 : s;
-            if (a.status) a.status[i] = err ? DC_ERR_INTERNAL : DC_OK;
-        }
-        for (int w = lane; w < W; w += 32) a.bits[i * W + w] = err ? 0u : bitsw[w];
-        __syncwarp();
+        __syncthreads();
     }
+    // release the slot, then finish no earlier than the previous launch of the
+    // batch, so that a kernel waiting for the last launch waits for them all
+    if (tid == 0) {
+        __threadfence();
+        atomicAnd(a.busy + slot_id / 32, ~(1u << (slot_id % 32)));
+    }
+    pdl_wait();
 }
 
 }  // namespace
@@ -616,54 +704,155 @@ __global__ void __launch_bounds__(32) deep_kernel(DeepArgs a)
 int sm_count();  // SMs of the current device (dp_small.cu)
 
 size_t deep_slot_bytes(int L) { return slot_bytes(L); }
-size_t deep_smem_bytes(int L) { return deep_smem(L); }
 
 // Resident one-warp CTAs per SM for depth L: a bound from shared memory alone
 // (the workspace is sized from it on the host, without a device query).
 int64_t deep_slots_bound(int L)
 {
-    const size_t per = deep_smem(L) + 1024;  // the runtime reserves 1 KB per CTA
+    const size_t per = deep_smem(L, 1) + 1024;  // the runtime reserves 1 KB per CTA
     int64_t n = int64_t((228 * 1024) / per);
     if (n > 32) n = 32;
     if (n < 1) n = 1;
     return 152 * n;
 }
 
-cudaError_t launch_deep(bool forward, int64_t lo, int64_t count, int L, const int64_t *comp,
-                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
-                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *ticket,
-                        uint32_t *list_count, uint32_t *list, void *slots, int64_t nslots,
-                        cudaStream_t stream)
+namespace {
+
+// Resident CTAs per SM of deep_kernel<FWD, NW> at depth L (raising the
+// kernel's shared-memory limit once per device first).
+template <bool FWD, int NW>
+cudaError_t deep_occupancy(int L, int &nb)
 {
-    if (count <= 0) return cudaSuccess;
-    const size_t smem = deep_smem(L);
-    static DeviceCache attr[2];  // the shared-memory limit, raised once per device and direction
+    static DeviceCache attr;
     int done = 0;
-    cudaError_t e = attr[forward ? 1 : 0].get(done, [&](int &v) {
-        const int most = int(deep_smem(DC_L_MAX));
+    cudaError_t e = attr.get(done, [](int &v) {
         v = 1;
-        return forward ? cudaFuncSetAttribute(deep_kernel<true>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize, most)
-                       : cudaFuncSetAttribute(deep_kernel<false>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        return cudaFuncSetAttribute(deep_kernel<FWD, NW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    int(deep_smem(DC_L_MAX, NW)));
     });
     if (e != cudaSuccess) return e;
-    int nb = 0;
-    e = forward ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, deep_kernel<true>, 32, smem)
-                : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, deep_kernel<false>, 32, smem);
-    if (e != cudaSuccess) return e;
-    int64_t grid = int64_t(sm_count()) * (nb > 0 ? nb : 1);
-    if (grid > nslots) grid = nslots;
-    if (grid > count) grid = count;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, deep_kernel<FWD, NW>, 32 * NW,
+                                                      deep_smem(L, NW));
+    if (nb < 1) nb = 1;
+    return e;
+}
+
+template <bool FWD, int NW>
+cudaError_t launch_deep_nw(const DeepArgs &a, int64_t grid, bool pdl, cudaStream_t stream)
+{
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(unsigned(grid));
+    lc.blockDim = dim3(32 * NW);
+    lc.dynamicSmemBytes = deep_smem(a.L, NW);
+    lc.stream = stream;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = at;
+    lc.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&lc, deep_kernel<FWD, NW>, a);
+}
+
+// Warps per instance. Persistent CTAs take instances in rounds of at most one
+// resident wave. An SM's throughput grows about linearly with its active warps
+// up to about 10 (measured: 10 one-warp instances per SM reach 0.78 of the
+// int-ALU roof, 4 about 0.23), and NW warps sharing an instance lose to their
+// per-column barrier and shorter blocks (about 0.7 / 0.6 / 0.55 of the one-warp
+// rate for 2 / 4 / 8 warps). Each choice's time is estimated round by round as
+// (instances per SM) / (min(active warps per SM, 10) x that efficiency), the
+// last round holding the remainder, and the smallest wins: one warp per
+// instance once the batch fills the GPU, more for a few hundred instances.
+template <bool FWD>
+cudaError_t launch_deep_dir(const DeepArgs &a, int64_t nslots, bool pdl, cudaStream_t stream)
+{
+    const int sms = sm_count();
+    const int nws[4] = {1, 2, 4, 8};
+    const double eta[4] = {1.0, 0.7, 0.6, 0.55};
+    int nb[4];
+    cudaError_t e;
+    if ((e = deep_occupancy<FWD, 1>(a.L, nb[0])) != cudaSuccess) return e;
+    if ((e = deep_occupancy<FWD, 2>(a.L, nb[1])) != cudaSuccess) return e;
+    if ((e = deep_occupancy<FWD, 4>(a.L, nb[2])) != cudaSuccess) return e;
+    if ((e = deep_occupancy<FWD, 8>(a.L, nb[3])) != cudaSuccess) return e;
+    int pick = 0;
+    int64_t grid_pick = 1;
+    double best = 0.0;
+    for (int q = 0; q < 4; ++q) {
+        int64_t G = int64_t(nb[q]) * sms;
+        if (G > nslots) G = nslots;
+        if (G > a.count) G = a.count;
+        double t = 0.0;
+        for (int64_t left = a.count; left > 0; left -= G) {
+            const double per_sm = double(left < G ? left : G) / sms;
+            const double active = per_sm * nws[q];
+            t += per_sm / ((active < 10.0 ? active : 10.0) * eta[q]);
+        }
+        if (q == 0 || t < best) {
+            best = t;
+            pick = q;
+            grid_pick = G;
+        }
+    }
+    switch (nws[pick]) {
+        case 1: return launch_deep_nw<FWD, 1>(a, grid_pick, pdl, stream);
+        case 2: return launch_deep_nw<FWD, 2>(a, grid_pick, pdl, stream);
+        case 4: return launch_deep_nw<FWD, 4>(a, grid_pick, pdl, stream);
+        default: return launch_deep_nw<FWD, 8>(a, grid_pick, pdl, stream);
+    }
+}
+
+}  // namespace
+
+// Instances per launch: about 90 ms of work at 0.67 of the int-ALU roof
+// (transitions C(L) per instance), and at least two resident waves of one-warp
+// CTAs, so that a long batch runs as launches of at most ~100 ms on a shared GPU.
+int64_t deep_per_launch(int64_t batch, int L)
+{
+    const double c = double(L) + double(L + 1) * double(L) * double(L - 1) / 6.0;
+    const double rate = 152.0 * 64.0 * 2.07e9 / 1.5 * 0.67;
+    int64_t per = int64_t(0.09 * rate / c);
+    const int64_t wave2 = 2 * deep_slots_bound(L);
+    if (per < wave2) per = wave2;
+    if (per >= batch) return batch;
+    const int64_t n = (batch + per - 1) / per;  // equal shares
+    return (batch + n - 1) / n;
+}
+
+int64_t deep_launches(int64_t batch, int L)
+{
+    if (batch <= 0) return 0;
+    const int64_t per = deep_per_launch(batch, L);
+    return (batch + per - 1) / per;
+}
+
+cudaError_t launch_deep(bool forward, int64_t batch, int L, const int64_t *comp,
+                        const int64_t *xfer, const int64_t *dt, int64_t *makespan,
+                        uint32_t *bits, int32_t *nseg, int32_t *status, uint32_t *tickets,
+                        uint32_t *busy, uint32_t *list_count, uint32_t *list, void *slots,
+                        int64_t nslots, cudaStream_t stream)
+{
+    if (batch <= 0) return cudaSuccess;
     const bool bulk = (L % 2 == 0) &&
                       ((reinterpret_cast<uintptr_t>(comp) | reinterpret_cast<uintptr_t>(xfer)) & 15u) == 0;
-    DeepArgs a{lo, count, L, comp, xfer, dt, makespan, bits, nseg, status, ticket, list_count, list,
-               static_cast<unsigned char *>(slots), slot_bytes(L), bulk ? 1 : 0};
-    if (forward)
-        deep_kernel<true><<<unsigned(grid), 32, smem, stream>>>(a);
-    else
-        deep_kernel<false><<<unsigned(grid), 32, smem, stream>>>(a);
-    return cudaGetLastError();
+    const int64_t per = deep_per_launch(batch, L);
+    // every launch's ticket and every slot's flag start at zero
+    cudaError_t e = cudaMemsetAsync(busy, 0, size_t((nslots + 31) / 32) * 4, stream);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(tickets, 0, size_t(deep_launches(batch, L)) * 4, stream);
+    if (e != cudaSuccess) return e;
+    int64_t k = 0;
+    for (int64_t lo = 0; lo < batch; lo += per, ++k) {
+        const int64_t count = batch - lo < per ? batch - lo : per;
+        DeepArgs a{lo, count, L, comp, xfer, dt, makespan, bits, nseg, status, tickets + k,
+                   list_count, list, busy, static_cast<unsigned char *>(slots), slot_bytes(L),
+                   int(nslots), bulk ? 1 : 0};
+        // the first launch waits for the memsets in stream order; later ones may
+        // overlap the tail of the one before
+        e = forward ? launch_deep_dir<true>(a, nslots, k > 0, stream)
+                    : launch_deep_dir<false>(a, nslots, k > 0, stream);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace dc

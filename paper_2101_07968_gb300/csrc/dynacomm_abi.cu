@@ -49,13 +49,15 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
     // warp-per-instance pass over the batch (three shifted 32-bit forms), then
     // the CTA-per-instance kernel over the instances it listed
     uint32_t *count = reinterpret_cast<uint32_t *>(ws);
-    uint32_t *ticket = count + 1;
     uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
-    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(uint32_t), stream);
+    const int64_t nslots = Workspace::deep_slots(batch, L);
+    uint32_t *busy = reinterpret_cast<uint32_t *>(ws + Workspace::table_offset(batch, L));
+    uint32_t *tickets = busy + nslots;
+    cudaError_t e = cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
     if (e != cudaSuccess) return e;
-    e = launch_deep(forward, 0, batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket,
-                    count, list, ws + Workspace::table_offset(batch, L),
-                    Workspace::deep_slots(batch, L), stream);
+    e = launch_deep(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, tickets,
+                    busy, count, list, ws + Workspace::deep_slots_offset(batch, L), nslots,
+                    stream);
     if (e != cudaSuccess) return e;
     return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, count,
                         list, ws + Workspace::group_tables_offset(batch, L),
@@ -119,6 +121,13 @@ dc_status dc_schedule_generated_batch(const dc_profile_cfg *cfg, int64_t *makesp
     return dc::launch_fused(g, makespan, bits, nseg, status, workspace, stream) == cudaSuccess
                ? DC_OK
                : DC_ERR_CUDA;
+}
+
+int32_t dc_schedule_kernel_launches(int64_t batch, int32_t L)
+{
+    if (batch <= 0 || L < 1 || L > DC_L_MAX) return 0;
+    if (L <= dc::kMidLMax) return 2;
+    return int32_t(dc::deep_launches(batch, L) + 1);
 }
 
 size_t dc_schedule_workspace_bytes(int64_t batch, int32_t L)

@@ -55,6 +55,7 @@ _VP, _I32, _I64, _SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c
 _SIGNATURES = {
     "dc_profile_gen": (_I32, [ctypes.POINTER(dc_profile_cfg), _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_schedule_workspace_bytes": (_SZ, [_I64, _I32]),
+    "dc_schedule_kernel_launches": (_I32, [_I64, _I32]),
     "dc_schedule_forward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
                                          _SZ, _VP]),
     "dc_schedule_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
@@ -126,6 +127,10 @@ def _check(st: int, what: str):
 # -------------------------------------------------------------- C ABI names
 def dc_status_string(status: int) -> str:
     return lib().dc_status_string(int(status)).decode()
+
+
+def dc_schedule_kernel_launches(batch: int, L: int) -> int:
+    return int(lib().dc_schedule_kernel_launches(int(batch), int(L)))
 
 
 def dc_schedule_workspace_bytes(batch: int, L: int) -> int:

@@ -64,6 +64,18 @@ def test_workspace_query(lib):
     assert dc.dc_schedule_workspace_bytes(16384, 1024) <= 5 * 2**30
 
 
+def test_kernel_launch_count(lib):
+    """Two passes per schedule call; long deep-chain batches split their first
+    pass into launches of about 90 ms of work (at least two resident waves)."""
+    f = dc.dc_schedule_kernel_launches
+    assert f(0, 16) == 0 and f(10, 0) == 0 and f(10, 4097) == 0
+    assert f(1_000_000, 16) == 2 and f(262_144, 54) == 2 and f(10, 256) == 2
+    assert f(1, 1024) == 2 and f(2000, 1024) == 2
+    deep = f(16384, 1024)
+    assert 3 <= deep <= 12          # 280 ms of work at the measured rate, split
+    assert f(32768, 1024) >= deep   # more work, at least as many launches
+
+
 FAKE = 0x1000  # never dereferenced: every case below fails its host check first
 
 

@@ -93,6 +93,31 @@ def test_dp_deep_random_parity(dc, L, kind):
         _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
 
 
+@pytest.mark.parametrize("B", [500, 1000, 2000])
+def test_dp_deep_warps_per_instance(dc, B):
+    """Batch sizes that give the deep-chain kernel 4, 2 and 1 warps per instance
+    (the rows of a column dealt to the warps strip by strip), full batches
+    bit-exact with the oracle; the xfer array starts 8 bytes past a 16-byte
+    boundary in one direction, which stages the rows with plain loads."""
+    import torch
+    L = 300
+    comp, xfer, dt = wl.skewed_instances(4000 + B, B, L)
+    buf = torch.empty(xfer.size + 1, dtype=torch.int64, device="cuda")
+    xs = buf[1:].view(xfer.shape)
+    xs.copy_(torch.from_numpy(xfer))
+    W = dc.words(L)
+    for d in (FWD, BWD):
+        if d == FWD:
+            got = _gpu_schedule(dc, d, comp, xfer, dt)
+        else:
+            out = dc.schedule(d, _dev(comp), xs, _dev(dt))
+            torch.cuda.synchronize()
+            got = {k: v.cpu().numpy() for k, v in out.items()}
+            got["bits"] = got["bits"].view(np.uint32)[:, :W]
+        exp = oracle.schedule_batch(d, comp, xfer, dt, nthreads=NTHREADS)
+        _assert_same(got, exp, f"B={B} dir={d}")
+
+
 @pytest.mark.parametrize("L", [1, 2, 8, 16, 17, 54, 70, 100, 200])
 def test_dp_wide_values_parity(dc, L):
     """Instances whose bound exceeds 2^32 need 64-bit arithmetic; mix them with
@@ -385,6 +410,23 @@ def test_config_deepchain_full_batch_digest(dc):
         bad = [(lo, hi) for (dd, lo, hi), h in sorted(want_chunks.items())
                if dd == d and mk.chunk_digest(got, lo, hi) != h]
         assert not bad, f"direction {d}: {len(bad)} chunks of 256 differ, first {bad[:4]}"
+
+
+def test_deepchain_split_launches_match_one_launch(dc):
+    """The full deep-chain batch runs as several chained launches (programmatic
+    dependent launch, per-launch tickets, claimed slots); its first 1,500
+    instances solved alone run as one launch. The outputs are bit-identical."""
+    import torch
+    assert dc.dc_schedule_kernel_launches(16384, 1024) > 2
+    assert dc.dc_schedule_kernel_launches(1500, 1024) == 2
+    prof = dc.profile_gen(wl.config("deepchain"))
+    for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
+        full = dc.schedule(d, prof[c], prof[x], prof["dt"])
+        part = dc.schedule(d, prof[c][:1500].contiguous(), prof[x][:1500].contiguous(),
+                           prof["dt"][:1500].contiguous())
+        torch.cuda.synchronize()
+        for k in ("makespan", "nseg", "status", "bits"):
+            assert torch.equal(full[k][:1500], part[k]), (d, k)
 
 
 @pytest.mark.parametrize("direction", [FWD, BWD])
