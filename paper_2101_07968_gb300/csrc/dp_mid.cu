@@ -44,8 +44,13 @@
 //    or 8 warps share a tile (same slices, less shared memory per warp): the
 //    column's row blocks are dealt to them in a snake, each warp keeps its
 //    results in registers until all have read column n-1 (a CTA barrier), then
-//    all write column n and meet at a second barrier. Warp 0 reads the rows and
-//    does the traceback.
+//    all write column n and meet at a second barrier. The tile's instances are
+//    dealt to the warps (32/NW each) for the row reads and the tracebacks, so
+//    no warp waits while another does them alone;
+//  * the traceback skips the candidates that cannot match: U[m] + V[k] is
+//    non-increasing in k and bounds the candidate from below, so a binary
+//    search over V finds the first k with U[m] + V[k] <= the cell, and the scan
+//    of the kept column starts there.
 #include "common.cuh"
 
 namespace dc {
@@ -267,7 +272,8 @@ __global__ void __launch_bounds__(32 * NW)
 {
     extern __shared__ uint32_t smem[];
     __shared__ uint32_t s_tile;
-    __shared__ int32_t s_dt[32];
+    __shared__ int32_t s_dt[32], s_fcL[32], s_go[32], s_best[32], s_s[32];
+    __shared__ uint64_t s_px[32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int W = words_for(L);
     // lane slices: U[v] at word 32*v + lane (v in [0, L]), then the current column
@@ -287,21 +293,27 @@ __global__ void __launch_bounds__(32 * NW)
         if (int64_t(tile) >= tiles) break;
         const int64_t i = int64_t(tile) * 32 + lane;
 
-        // ---- rows -> lane slices (warp 0)
-        bool go = false;
-        uint64_t px = 0;
-        int32_t fcL = 0;
-        if (warp == 0) {
+        // ---- rows -> lane slices: the tile's instances dealt to the warps, 32/NW
+        // each (a lane's slice is the same in every warp)
+        const bool mine = lane / (32 / NW) == warp;
+        if (mine) {
             const int64_t dti = i < batch ? __ldg(dt + i) : 0;
-            go = i < batch && mid_prefix<FWD>(i, L, comp, xfer, dti, lw, pv, makespan, bits,
-                                              nseg, status, list_count, list, px, fcL);
+            uint64_t px = 0;
+            int32_t fcL = 0;
+            const bool go = i < batch && mid_prefix<FWD>(i, L, comp, xfer, dti, lw, pv, makespan,
+                                                         bits, nseg, status, list_count, list, px,
+                                                         fcL);
             s_dt[lane] = int32_t(dti);
+            s_go[lane] = go;
+            s_px[lane] = px;
+            s_fcL[lane] = fcL;
         }
-        if (NW > 1) __syncthreads();
+        if (NW > 1) __syncthreads(); else __syncwarp();
         // every lane runs the fill (lanes without an instance on stale slices:
         // all accesses stay in the lane's own slice and slot), so that the
         // barriers of the split fill are reached by all threads
         const int32_t dt32 = s_dt[lane];
+        const int32_t fcL = s_fcL[lane];
 
         // ---- fill
         int32_t bestV = 0;
@@ -354,7 +366,16 @@ __global__ void __launch_bounds__(32 * NW)
                 }
             }
         }
-        if (warp != 0 || !go) continue;
+        // the tracebacks, dealt to the warps like the rows
+        if (warp == 0) {
+            s_best[lane] = bestV;
+            s_s[lane] = s;
+        }
+        if (NW > 1) __syncthreads(); else __syncwarp();
+        if (!mine || !s_go[lane]) continue;
+        bestV = s_best[lane];
+        s = s_s[lane];
+        const uint64_t px = s_px[lane];
         if (s - 1 > keep && s - 1 >= 2) {  // traceback would need an unkept column
             list[atomicAdd(list_count, 1u)] = uint32_t(i);
             continue;
@@ -368,10 +389,22 @@ __global__ void __launch_bounds__(32 * NW)
         int32_t target = FWD ? bestV - s * dt32 + U[32 * L] : bestV - 2 * dt32;  // B[L][s] + Q[L] or F[L][s] - dt
         while (n > 1) {
             const int32_t uu = U[32 * m];
+            // U[m] + V[k] is non-increasing in k (V is G forward, the negated
+            // transfer prefix backward) and a candidate max(U[m] + V[k], C[k]) is
+            // at least U[m] + V[k]: every k before the first with U[m] + V[k] <=
+            // target misses, and the scan starts there
+            int lo = n - 1, hi = m - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (uu + pv[32 * mid].y > target)
+                    lo = mid + 1;
+                else
+                    hi = mid;
+            }
             // candidates in groups of 8 (loads issued together, lowest match wins)
             int k = -1;
             int32_t fk = 0;
-            for (int k0 = n - 1; k0 < m && k < 0; k0 += 8) {
+            for (int k0 = lo; k0 < m && k < 0; k0 += 8) {
                 int32_t f[8], v[8];
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
