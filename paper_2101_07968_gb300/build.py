@@ -20,6 +20,9 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdynacomm.so")
+# the checked build (-DDC_CHECKED): index checks that count failures instead of trapping
+LIB_CHECKED = os.path.join(PKG, "libdynacomm_checked.so")
+BUILD_CHECKED = os.path.join(PKG, "_build_checked")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
@@ -49,19 +52,23 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile and link if any source is newer than the library. Returns its path."""
+def build(force: bool = False, verbose: bool = False, checked: bool = False) -> str:
+    """Compile and link if any source is newer than the library. Returns its path.
+    checked=True builds libdynacomm_checked.so with -DDC_CHECKED instead."""
+    lib_path = LIB_CHECKED if checked else LIB
+    build_dir = BUILD_CHECKED if checked else BUILD
+    flags = NVCC_FLAGS + (["-DDC_CHECKED"] if checked else [])
     deps = _deps()
-    if not force and not _stale(LIB, deps):
-        return LIB
-    os.makedirs(BUILD, exist_ok=True)
+    if not force and not _stale(lib_path, deps):
+        return lib_path
+    os.makedirs(build_dir, exist_ok=True)
     exe = nvcc()
     headers = glob.glob(os.path.join(CSRC, "*.cuh")) + [os.path.join(INCLUDE, "dynacomm.h")]
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         if force or _stale(obj, [src] + headers + [os.path.abspath(__file__)]):
-            cmd = [exe, "-c", src, "-o", obj] + NVCC_FLAGS
+            cmd = [exe, "-c", src, "-o", obj] + flags
             if verbose:
                 cmd += ["-Xptxas", "-v"]
             res = subprocess.run(cmd, capture_output=True, text=True)
@@ -73,7 +80,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
 
     with ThreadPoolExecutor(max_workers=max(2, os.cpu_count() or 2)) as ex:
         objs = list(ex.map(compile_one, _sources()))
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib_path + f".tmp{os.getpid()}"
     # Shared CUDA runtime (soname libcudart.so.13): when torch has loaded its copy
     # first, the loader reuses it, so both see one current device and one
     # default stream. The rpath finds the toolkit's copy otherwise.
@@ -83,9 +90,10 @@ def build(force: bool = False, verbose: bool = False) -> str:
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv,
+                checked="--checked" in sys.argv))

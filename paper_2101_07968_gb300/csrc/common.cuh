@@ -6,6 +6,7 @@
 #include <mutex>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "dynacomm.h"
 
@@ -97,6 +98,52 @@ struct Workspace {
     {
         return group_tables_offset(batch, L) + slots(batch, L) * size_t(tri_cells(L)) * 8;
     }
+};
+
+// Index checks of the checked build (compiled with -DDC_CHECKED): a check that
+// fails counts itself in this translation unit's device counters (the first
+// failing source line is kept) and the caller skips the access; nothing traps.
+// dc_checked_<unit>() reads (and optionally clears) a unit's counters from the
+// host. In the normal build DC_CHECK(cond) is `true` and costs nothing.
+#ifdef DC_CHECKED
+namespace {
+__device__ unsigned int g_check_count;
+__device__ unsigned int g_check_line;
+__device__ __noinline__ bool check_failed(unsigned line)
+{
+    if (atomicAdd(&g_check_count, 1u) == 0u) atomicExch(&g_check_line, line);
+    return false;
+}
+}  // namespace
+#define DC_CHECK(cond) ((cond) ? true : ::dc::check_failed(__LINE__))
+#define DC_CHECKED_EXPORT(unit)                                                                \
+    extern "C" int dc_checked_##unit(unsigned int *count, unsigned int *line, int reset)       \
+    {                                                                                          \
+        if (cudaMemcpyFromSymbol(count, ::dc::g_check_count, sizeof(unsigned int)) !=          \
+                cudaSuccess ||                                                                 \
+            cudaMemcpyFromSymbol(line, ::dc::g_check_line, sizeof(unsigned int)) != cudaSuccess) \
+            return -1;                                                                         \
+        if (reset) {                                                                           \
+            const unsigned int z = 0u;                                                         \
+            if (cudaMemcpyToSymbol(::dc::g_check_count, &z, sizeof z) != cudaSuccess ||        \
+                cudaMemcpyToSymbol(::dc::g_check_line, &z, sizeof z) != cudaSuccess)           \
+                return -1;                                                                     \
+        }                                                                                      \
+        return 0;                                                                              \
+    }
+#else
+#define DC_CHECK(cond) true
+#define DC_CHECKED_EXPORT(unit)
+#endif
+
+// An NVTX range over one C-ABI call: named on the timelines of Nsight Systems
+// and Nsight Compute when a tool is attached, a few instructions otherwise
+// (header-only NVTX 3; it loads no library unless a tool asks).
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
 };
 
 // A per-device launch fact (resident CTAs per SM of a kernel, the SM count),

@@ -178,6 +178,11 @@ __device__ __forceinline__ void block(int L, int n, int b0, int k_lo, bool far, 
                                       const int32_t *__restrict__ urow, int32_t *__restrict__ kept,
                                       int32_t *__restrict__ last, int koff, int lane)
 {
+    // the block's pair entries (from k_lo - 1 to its top) and rows lie inside
+    // the arrays
+    if (!DC_CHECK(k_lo - 1 + koff >= 0 && b0 + koff >= 0 && b0 + S * (R - 1) + 31 <= L &&
+                  b0 + S * (R - 1) + 31 + koff < deep_entries(L)))
+        return;
     int32_t u[R], acc[R];
     const int32_t ndt1 = (FORM == kS32 && !FWD) ? int32_t(int64_t(n - 1) * dt) : 0;
 #pragma unroll
@@ -258,7 +263,7 @@ __device__ __forceinline__ void block(int L, int n, int b0, int k_lo, bool far, 
             ny = c.y;
         }
         nxt[m + koff] = make_int2(nx, ny);
-        if (n <= kKeep) kept[tri_index(L, m, n)] = X;
+        if (n <= kKeep && DC_CHECK(tri_index(L, m, n) < kept_cells(L))) kept[tri_index(L, m, n)] = X;
         if (m == L) last[n] = X;
     }
 }
@@ -370,6 +375,7 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
     }
     __syncthreads();
     const int slot_id = reinterpret_cast<volatile int32_t *>(smem + 8)[1];
+    if (!DC_CHECK(slot_id < a.nslots)) return;
     if (slot_id < 0) {  // every slot held (not expected): leave the instances to the other CTAs
         pdl_wait();
         return;
@@ -481,7 +487,10 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
                     else
                         flag = kListed;
                     if (flag == kListed) {  // 32/64-bit literal template: the CTA-per-instance kernel
-                        if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+                        if (lane == 0) {
+                            const uint32_t at = atomicAdd(a.list_count, 1u);
+                            if (DC_CHECK(int64_t(at) < a.lo + a.count)) a.list[at] = uint32_t(i);
+                        }
                     } else {
                         // prefix sums in processing order: comp (below 2^31) into
                         // urow, capped transfers (64-bit) into the slot
@@ -597,7 +606,10 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
         bool planned = true;
         for (int w = 0; w < NW; ++w) planned &= plans[w * (PM + 1) + PM].x >= 0;
         if (!planned) {  // blocks narrower than one strip: the CTA-per-instance kernel
-            if (tid == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+            if (tid == 0) {
+                            const uint32_t at = atomicAdd(a.list_count, 1u);
+                            if (DC_CHECK(int64_t(at) < a.lo + a.count)) a.list[at] = uint32_t(i);
+                        }
             __syncthreads();
             continue;
         }
@@ -635,7 +647,10 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
             }
             const int s = bn;
             if (s - 1 > kKeep) {  // the traceback needs columns beyond the kept ones
-                if (lane == 0) a.list[atomicAdd(a.list_count, 1u)] = uint32_t(i);
+                if (lane == 0) {
+                            const uint32_t at = atomicAdd(a.list_count, 1u);
+                            if (DC_CHECK(int64_t(at) < a.lo + a.count)) a.list[at] = uint32_t(i);
+                        }
             } else {
                 // Path[m][n] = the lowest k whose candidate equals the cell
                 int err = 0, m = L, n = s;
@@ -648,7 +663,7 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
                         const int k = k0 + lane;
                         bool match = false;
                         if (k < m) {
-                            const int32_t Xk = kept[pbase + k];
+                            const int32_t Xk = DC_CHECK(pbase + k < kept_cells(L)) ? kept[pbase + k] : 0;
                             if (form == kS32) {
                                 const int32_t u = FWD ? urow[m] : urow[m] - int32_t(int64_t(n - 1) * dti);
                                 const int32_t target = FWD ? Xmn + int32_t(dti) : Xmn;
@@ -856,3 +871,5 @@ cudaError_t launch_deep(bool forward, int64_t batch, int L, const int64_t *comp,
 }
 
 }  // namespace dc
+
+DC_CHECKED_EXPORT(dp_deep)

@@ -76,7 +76,8 @@ __device__ __forceinline__ void fused_direction(const GenParams &g, const GenTab
         write_failure(st, i, W, o.makespan[dir], o.bits[dir], o.nseg[dir], o.status[dir]);
     } else if (wide || !solve_uv<L, FWD>(U, V, int32_t(dti), xraw, lw, i, o.makespan[dir],
                                          o.bits[dir], o.nseg[dir], o.status[dir])) {
-        o.wide_list[dir][atomicAdd(o.wide_count[dir], 1u)] = uint32_t(i);
+        const uint32_t at = atomicAdd(o.wide_count[dir], 1u);
+        if (DC_CHECK(int64_t(at) < g.batch)) o.wide_list[dir][at] = uint32_t(i);
     }
 }
 
@@ -237,3 +238,5 @@ cudaError_t launch_fused(const GenParams &g, int64_t *makespan, uint32_t *bits, 
 }
 
 }  // namespace dc
+
+DC_CHECKED_EXPORT(dp_fused)

@@ -219,7 +219,7 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
         const T v = T(R + S[skew(m)] + c);
         colA[skew(m)] = v;
         best[skew(m)] = T(~T(0));
-        table[tri_index(L, m, 1)] = v;
+        if (DC_CHECK(tri_index(L, m, 1) < tri_cells(L))) table[tri_index(L, m, 1)] = v;
     }
     __syncthreads();
     T *prev = colA, *cur = colB;
@@ -231,7 +231,7 @@ __device__ void solve(const GroupArgs &a, int64_t i, int64_t dti, uint64_t shift
             const T v = T(best[skew(m)] + S[skew(m)] + c);
             cur[skew(m)] = v;
             best[skew(m)] = T(~T(0));
-            table[cbase + m] = v;
+            if (DC_CHECK(cbase + m < tri_cells(L))) table[cbase + m] = v;
         }
         __syncthreads();
         T *tmp = prev;
@@ -403,7 +403,7 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
         const int32_t v = FWD ? fcL + U[skew(m)] - dt : U[skew(m)];
         colA[skew(m)] = v;
         best[skew(m)] = 0x7fffffff;
-        table[tri_index(L, m, 1)] = v;
+        if (DC_CHECK(tri_index(L, m, 1) < tri_cells(L))) table[tri_index(L, m, 1)] = v;
     }
     __syncthreads();
     int32_t *prev = colA, *cur = colB;
@@ -416,7 +416,7 @@ __device__ void solve_s32(const GroupArgs &a, int64_t i, int64_t dti, uint64_t x
             const int32_t v = FWD ? b - dt : b;
             cur[skew(m)] = v;
             best[skew(m)] = 0x7fffffff;
-            table[cbase + m] = v;
+            if (DC_CHECK(cbase + m < tri_cells(L))) table[cbase + m] = v;
         }
         __syncthreads();
         int32_t *tmp = prev;
@@ -571,7 +571,7 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
         const int32_t v = BC[skew(m)];
         colA[skew(m)] = v;
         best[skew(m)] = 0x7fffffff;
-        table[tri_index(L, m, 1)] = v;
+        if (DC_CHECK(tri_index(L, m, 1) < tri_cells(L))) table[tri_index(L, m, 1)] = v;
         NY[skew(m)] = -yclamp(dtv + GT[skew(m)]);
     }
     __syncthreads();
@@ -584,7 +584,7 @@ __device__ void solve_ebwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
             const int32_t v = best[skew(m)];
             cur[skew(m)] = v;
             best[skew(m)] = 0x7fffffff;
-            table[cbase + m] = v;
+            if (DC_CHECK(cbase + m < tri_cells(L))) table[cbase + m] = v;
         }
         for (int k = n + t; k <= L; k += nt) NY[skew(k)] = -yclamp(uint64_t(n) * dtv + GT[skew(k)]);
         __syncthreads();
@@ -786,7 +786,7 @@ __device__ void solve_efwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
         const int32_t v = int32_t(fcL) - G[skew(m)];
         colA[skew(m)] = v;
         best[skew(m)] = 0x7fffffff;
-        table[tri_index(L, m, 1)] = v;
+        if (DC_CHECK(tri_index(L, m, 1) < tri_cells(L))) table[tri_index(L, m, 1)] = v;
         A[skew(m)] = fcL + P[skew(m)];
     }
     __syncthreads();
@@ -800,7 +800,7 @@ __device__ void solve_efwd(const GroupArgs &a, int64_t i, int64_t dti, uint64_t 
             const int32_t v = bm - G[skew(m)];
             cur[skew(m)] = v;
             best[skew(m)] = 0x7fffffff;
-            table[cbase + m] = v;
+            if (DC_CHECK(cbase + m < tri_cells(L))) table[cbase + m] = v;
             A[skew(m)] = uint64_t(bm) + P[skew(m)];  // E + G + P for column n+1
         }
         __syncthreads();
@@ -887,6 +887,7 @@ __global__ void __launch_bounds__(256) group_kernel(GroupArgs a)
     const int64_t count = a.list_count ? int64_t(*a.list_count) : a.batch;
     for (int64_t j = blockIdx.x; j < count; j += gridDim.x) {
         const int64_t i = a.list ? int64_t(a.list[j]) : j;
+        if (!DC_CHECK(i >= 0 && i < a.batch)) continue;
         const int64_t *crow = a.comp + i * L;
         const int64_t *xrow = a.xfer + i * L;
         const int64_t dti = a.dt[i];
@@ -1000,3 +1001,5 @@ cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp
 }
 
 }  // namespace dc
+
+DC_CHECKED_EXPORT(dp_group)

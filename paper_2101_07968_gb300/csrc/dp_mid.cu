@@ -97,7 +97,7 @@ __host__ __device__ inline int64_t mid_slots(int64_t batch, int L)
 // (an input error, whose outputs it writes, or values beyond 31 bits, which it
 // lists for the CTA-per-instance kernel).
 template <bool FWD>
-__device__ __forceinline__ bool mid_prefix(int64_t i, int L, const int64_t *__restrict__ comp,
+__device__ __forceinline__ bool mid_prefix(int64_t batch, int64_t i, int L, const int64_t *__restrict__ comp,
                                            const int64_t *__restrict__ xfer, int64_t dti,
                                            uint32_t *lw, int2 *pv, int64_t *makespan,
                                            uint32_t *bits, int32_t *nseg, int32_t *status,
@@ -142,7 +142,10 @@ __device__ __forceinline__ bool mid_prefix(int64_t i, int L, const int64_t *__re
                                int32_t(FWD ? tcu - uint32_t(pc) : 0u - uint32_t(pxc)));
     }
     if (pc + pxc + uint64_t(L) * uint64_t(dti) > kShiftedLimit) {
-        list[atomicAdd(list_count, 1u)] = uint32_t(i);
+        {
+            const uint32_t at = atomicAdd(list_count, 1u);
+            if (DC_CHECK(int64_t(at) < batch)) list[at] = uint32_t(i);
+        }
         return false;
     }
     fcL = int32_t(tcu);
@@ -222,6 +225,8 @@ __device__ __forceinline__ void mid_write(int2 *pv, uint32_t *myslot, int64_t ns
                                           const int32_t (&best)[kB], int32_t dt32, int32_t &last)
 {
     const int64_t cb = int64_t(mid_cell(L, bot, n)) * nslots;
+    // the kept cells of rows bot..top (column n <= keep) lie in the slot's cells
+    if (!DC_CHECK(n > keep || (bot >= n && top <= L && mid_cell(L, top, n) < mid_cells(L)))) return;
     if (top - bot == kB - 1) {  // full block
 #pragma unroll
         for (int j = 0; j < kB; ++j) {
@@ -300,7 +305,7 @@ __global__ void __launch_bounds__(32 * NW)
             const int64_t dti = i < batch ? __ldg(dt + i) : 0;
             uint64_t px = 0;
             int32_t fcL = 0;
-            const bool go = i < batch && mid_prefix<FWD>(i, L, comp, xfer, dti, lw, pv, makespan,
+            const bool go = i < batch && mid_prefix<FWD>(batch, i, L, comp, xfer, dti, lw, pv, makespan,
                                                          bits, nseg, status, list_count, list, px,
                                                          fcL);
             s_dt[lane] = int32_t(dti);
@@ -377,7 +382,10 @@ __global__ void __launch_bounds__(32 * NW)
         s = s_s[lane];
         const uint64_t px = s_px[lane];
         if (s - 1 > keep && s - 1 >= 2) {  // traceback would need an unkept column
-            list[atomicAdd(list_count, 1u)] = uint32_t(i);
+            {
+            const uint32_t at = atomicAdd(list_count, 1u);
+            if (DC_CHECK(int64_t(at) < batch)) list[at] = uint32_t(i);
+        }
             continue;
         }
 
@@ -413,7 +421,9 @@ __global__ void __launch_bounds__(32 * NW)
                     if (n - 1 == 1)  // column 1 from U
                         f[u] = FWD ? fcL + U[32 * kk] - dt32 : U[32 * kk] + dt32;
                     else
-                        f[u] = int32_t(myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots]);
+                        f[u] = DC_CHECK(mid_cell(L, kk, n - 1) < mid_cells(L))
+                                   ? int32_t(myslot[int64_t(mid_cell(L, kk, n - 1)) * nslots])
+                                   : 0;
                 }
 #pragma unroll
                 for (int u = 8 - 1; u >= 0; --u) {
@@ -496,3 +506,5 @@ cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
 }
 
 }  // namespace dc
+
+DC_CHECKED_EXPORT(dp_mid)

@@ -101,7 +101,8 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         } else if (wide ||
                    !solve_uv<L, FWD>(U, V, int32_t(dti), xraw, lw, i, makespan, bits, nseg, status)) {
             // 64-bit values, or a traceback deeper than the kept columns: work list
-            wide_list[atomicAdd(wide_count, 1u)] = uint32_t(i);
+            const uint32_t at = atomicAdd(wide_count, 1u);
+            if (DC_CHECK(int64_t(at) < batch)) wide_list[at] = uint32_t(i);
         }
     }
 }
@@ -231,3 +232,5 @@ cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp
 }
 
 }  // namespace dc
+
+DC_CHECKED_EXPORT(dp_small)

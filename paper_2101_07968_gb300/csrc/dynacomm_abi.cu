@@ -89,6 +89,7 @@ extern "C" {
 dc_status dc_profile_gen(const dc_profile_cfg *cfg, int64_t *fc, int64_t *pt, int64_t *bc,
                          int64_t *gt, int64_t *dt, cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_profile_gen");
     if (!cfg) return DC_ERR_NULL;
     const dc_status st = dc::check_profile_cfg(cfg);
     if (st != DC_OK) return st;
@@ -108,6 +109,7 @@ dc_status dc_schedule_generated_batch(const dc_profile_cfg *cfg, int64_t *makesp
                                       void *workspace, size_t workspace_bytes,
                                       cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_schedule_generated_batch");
     if (!cfg) return DC_ERR_NULL;
     const dc_status st = dc::check_profile_cfg(cfg);
     if (st != DC_OK) return st;
@@ -141,6 +143,7 @@ dc_status dc_schedule_forward_batch(int64_t batch, int32_t L, const int64_t *fc,
                                     uint32_t *bits, int32_t *nseg, int32_t *status,
                                     void *workspace, size_t workspace_bytes, cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_schedule_forward_batch");
     return dc::schedule(true, batch, L, fc, pt, dt, makespan, bits, nseg, status, workspace,
                         workspace_bytes, stream);
 }
@@ -151,6 +154,7 @@ dc_status dc_schedule_backward_batch(int64_t batch, int32_t L, const int64_t *bc
                                      void *workspace, size_t workspace_bytes,
                                      cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_schedule_backward_batch");
     return dc::schedule(false, batch, L, bc, gt, dt, makespan, bits, nseg, status, workspace,
                         workspace_bytes, stream);
 }
@@ -159,6 +163,7 @@ dc_status dc_eval_timeline_batch(int64_t batch, int32_t L, int32_t dir, const in
                                  const int64_t *xfer, const int64_t *dt, const uint32_t *bits,
                                  int64_t *makespan, cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_eval_timeline_batch");
     if (batch < 0 || L < 1 || L > DC_L_MAX || (dir != 0 && dir != 1)) return DC_ERR_BAD_SHAPE;
     if (batch == 0) return DC_OK;
     if (!comp || !xfer || !dt || !makespan || (!bits && dc::words_for(L) > 0))
@@ -188,6 +193,7 @@ const char *dc_status_string(dc_status s)
 dc_status dc_roof_int_probe(int32_t variant, int32_t blocks, int32_t threads, int64_t iters,
                             uint32_t *sink, cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_roof_int_probe");
     if (variant != 0 && variant != 1) return DC_ERR_BAD_SHAPE;
     if (blocks < 1 || threads < 32 || threads > 1024 || threads % 32 || iters < 0 || iters % 4)
         return DC_ERR_BAD_SHAPE;

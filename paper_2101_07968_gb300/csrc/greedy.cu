@@ -256,6 +256,7 @@ extern "C" dc_status dc_greedy_forward_batch(int64_t batch, int32_t L, const int
                                              int64_t *makespan, uint32_t *bits,
                                              cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_greedy_forward_batch");
     if (batch < 0 || L < 1 || L > DC_L_MAX || batch > int64_t(0xffffffffll)) return DC_ERR_BAD_SHAPE;
     if (batch == 0) return DC_OK;
     if (!fc || !pt || !dt || !makespan || (!bits && dc::words_for(L) > 0)) return DC_ERR_NULL;
@@ -269,6 +270,7 @@ extern "C" dc_status dc_greedy_backward_batch(int64_t batch, int32_t L, const in
                                               int64_t *makespan, uint32_t *bits,
                                               cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_greedy_backward_batch");
     if (batch < 0 || L < 1 || L > DC_L_MAX || batch > int64_t(0xffffffffll)) return DC_ERR_BAD_SHAPE;
     if (batch == 0) return DC_OK;
     if (!bc || !gt || !dt || !makespan || (!bits && dc::words_for(L) > 0)) return DC_ERR_NULL;

@@ -51,6 +51,7 @@ extern "C" dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_
                                               uint32_t *bits, int32_t *nseg, int32_t *status,
                                               cudaStream_t stream)
 {
+    const dc::NvtxRange nvtx("dc_schedule_batch_static");
     if ((dir != 0 && dir != 1) || batch < 0 || L < 1 || L > dc::kSmallLMax)
         return DC_ERR_BAD_SHAPE;
     if (batch > dc::kStaticMaxBatch) return DC_ERR_WORKSPACE;  // beyond the static scratch

@@ -17,7 +17,11 @@ import os
 from typing import Optional
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libdynacomm.so")
+# DC_CHECKED=1 loads the checked build (index checks that count failures
+# instead of trapping; build it with `python -m paper_2101_07968_gb300.build --checked`)
+LIB_PATH = os.path.join(_PKG, "libdynacomm_checked.so" if os.environ.get("DC_CHECKED") == "1"
+                        else "libdynacomm.so")
+CHECKED_UNITS = ("dp_deep", "dp_mid", "dp_small", "dp_group", "dp_fused")
 
 DC_OK, DC_ERR_NULL, DC_ERR_BAD_SHAPE, DC_ERR_NEGATIVE, DC_ERR_RANGE = 0, 1, 2, 3, 4
 DC_ERR_WORKSPACE, DC_ERR_CUDA, DC_ERR_BAD_CONFIG, DC_ERR_INTERNAL = 5, 6, 7, 8
@@ -91,6 +95,25 @@ def lib():
 
 def exported_names():
     return list(_SIGNATURES)
+
+
+def checked_failures(reset: bool = False) -> dict:
+    """Index-check counters of the checked build, per translation unit:
+    {unit: (failed checks, source line of the first)}. reset=True clears them.
+    Raises if the loaded library is not the checked build."""
+    l = lib()
+    out = {}
+    for unit in CHECKED_UNITS:
+        fn = getattr(l, "dc_checked_" + unit, None)
+        if fn is None:
+            raise RuntimeError(f"{LIB_PATH} is not the checked build")
+        fn.restype = ctypes.c_int
+        fn.argtypes = [ctypes.POINTER(ctypes.c_uint), ctypes.POINTER(ctypes.c_uint), ctypes.c_int]
+        count, line = ctypes.c_uint(0), ctypes.c_uint(0)
+        if fn(ctypes.byref(count), ctypes.byref(line), int(reset)) != 0:
+            raise RuntimeError(f"reading the check counters of {unit} failed")
+        out[unit] = (int(count.value), int(line.value))
+    return out
 
 
 # ------------------------------------------------------------- marshalling
