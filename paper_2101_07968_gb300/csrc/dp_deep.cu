@@ -70,10 +70,13 @@ __host__ __device__ inline int deep_koff(int L) { return kPad + ((L + 1) & 1); }
 __host__ __device__ inline int deep_entries(int L) { return L + kPad + 2; }
 __host__ __device__ inline size_t deep_pair_bytes(int L) { return al16(size_t(deep_entries(L)) * 8); }
 __host__ __device__ inline int deep_plan_max(int L) { return L / 32 + 2; }
-__host__ __device__ inline size_t deep_urow_off(int L) { return 16 + 2 * deep_pair_bytes(L); }
-__host__ __device__ inline size_t deep_bits_off(int L) { return deep_urow_off(L) + al16(size_t(L + 1) * 4); }
-__host__ __device__ inline size_t deep_plan_off(int L) { return deep_bits_off(L) + al16(size_t(words_for(L) + 1) * 4); }
-__host__ __device__ inline size_t deep_smem(int L, int NW) { return deep_plan_off(L) + size_t(NW) * (deep_plan_max(L) + 1) * 16; }
+// One pair buffer with one warp per instance (the column is updated in place:
+// blocks run top-down and read only rows below their own top), two otherwise.
+__host__ __device__ inline int deep_buffers(int NW) { return NW == 1 ? 1 : 2; }
+__host__ __device__ inline size_t deep_urow_off(int L, int NW) { return 16 + deep_buffers(NW) * deep_pair_bytes(L); }
+__host__ __device__ inline size_t deep_bits_off(int L, int NW) { return deep_urow_off(L, NW) + al16(size_t(L + 1) * 4); }
+__host__ __device__ inline size_t deep_plan_off(int L, int NW) { return deep_bits_off(L, NW) + al16(size_t(words_for(L) + 1) * 4); }
+__host__ __device__ inline size_t deep_smem(int L, int NW) { return deep_plan_off(L, NW) + size_t(NW) * (deep_plan_max(L) + 1) * 16; }
 
 __host__ __device__ inline int64_t kept_cols(int L) { return L < kKeep ? L : kKeep; }
 __host__ __device__ inline int64_t kept_cells(int L)
@@ -341,10 +344,10 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
     uint64_t *bar = reinterpret_cast<uint64_t *>(smem);
     volatile int32_t *ctl = reinterpret_cast<volatile int32_t *>(smem + 8);  // instance, flag
     int2 *XY0 = reinterpret_cast<int2 *>(smem + 16);
-    int2 *XY1 = reinterpret_cast<int2 *>(smem + 16 + deep_pair_bytes(L));
-    int32_t *urow = reinterpret_cast<int32_t *>(smem + deep_urow_off(L));
-    uint32_t *bitsw = reinterpret_cast<uint32_t *>(smem + deep_bits_off(L));
-    int4 *plans = reinterpret_cast<int4 *>(smem + deep_plan_off(L));
+    int2 *XY1 = reinterpret_cast<int2 *>(smem + 16 + (deep_buffers(NW) - 1) * deep_pair_bytes(L));
+    int32_t *urow = reinterpret_cast<int32_t *>(smem + deep_urow_off(L, NW));
+    uint32_t *bitsw = reinterpret_cast<uint32_t *>(smem + deep_bits_off(L, NW));
+    int4 *plans = reinterpret_cast<int4 *>(smem + deep_plan_off(L, NW));
     int4 *plan = plans + warp * (PM + 1);
 
     // The next launch of a split batch may start filling SMs as this one's CTAs
@@ -385,8 +388,7 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
     int32_t *last = reinterpret_cast<int32_t *>(slot + slot_last_off(L));
     int32_t *Gk = reinterpret_cast<int32_t *>(slot + slot_g_off(L));
     int32_t *kept = reinterpret_cast<int32_t *>(slot + slot_kept_off(L));
-    uint64_t *rawc = reinterpret_cast<uint64_t *>(XY0);
-    uint64_t *rawx = reinterpret_cast<uint64_t *>(XY1);
+    uint64_t *raw = reinterpret_cast<uint64_t *>(XY0);  // one profile row at a time
 
     if (a.bulk && tid == 0) mbar_init(bar);
     __syncthreads();
@@ -408,51 +410,72 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
         // ---- warp 0: rows, checks, form, prefix sums, column 1
         if (warp == 0) {
             int flag = 0;
-            bool staged = true;
-            if (a.bulk) {
+            // one profile row into the staging buffer: 0 landed, 1 lost (the
+            // instance is marked failed), 2 lost and perhaps still in flight
+            auto stage = [&](const int64_t *row) -> int {
+                if (!a.bulk) {
+                    for (int c = lane; c < L; c += 32) raw[c] = uint64_t(__ldg(row + c));
+                    __syncwarp();
+                    return 0;
+                }
+                // the buffer's earlier reads and writes before the copy's writes
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) {
-                    mbar_expect(bar, uint32_t(16) * uint32_t(L));
-                    bulk_g2s(rawc, a.comp + i * L, uint32_t(8) * uint32_t(L), bar);
-                    bulk_g2s(rawx, a.xfer + i * L, uint32_t(8) * uint32_t(L), bar);
+                    mbar_expect(bar, uint32_t(8) * uint32_t(L));
+                    bulk_g2s(raw, row, uint32_t(8) * uint32_t(L), bar);
                 }
                 const bool ok = mbar_wait(bar, phase, 1 << 22);
                 phase ^= 1u;
-                if (!__all_sync(0xffffffffu, ok)) {
-                    // the copies did not land in time: wait once more before the
-                    // buffers are given up, then leave the instance failed
-                    const bool late = mbar_wait(bar, phase ^ 1u, 1 << 22);
-                    if (lane == 0) {
-                        a.makespan[i] = -int64_t(DC_ERR_INTERNAL);
-                        if (a.nseg) a.nseg[i] = 0;
-                        if (a.status) a.status[i] = DC_ERR_INTERNAL;
-                    }
-                    for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
-                    staged = false;
-                    flag = __all_sync(0xffffffffu, late) ? int(kListed) : int(kAbort);
-                }
-            } else {
-                for (int c = lane; c < L; c += 32) {
-                    rawc[c] = uint64_t(__ldg(a.comp + i * L + c));
-                    rawx[c] = uint64_t(__ldg(a.xfer + i * L + c));
-                }
-                __syncwarp();
-            }
-            if (staged) {
-                bool neg = dti < 0, big = (dti >> 52) != 0;
-                uint64_t sc = 0;
+                if (__all_sync(0xffffffffu, ok)) return 0;
+                // the copy did not land in time: wait once more before the buffer
+                // is given up
+                const bool late = mbar_wait(bar, phase ^ 1u, 1 << 22);
+                return __all_sync(0xffffffffu, late) ? 1 : 2;
+            };
+            // compute row: checks, total, prefix (wrapping; used only when the
+            // total is below 2^31) into urow
+            int lost = stage(a.comp + i * L);
+            bool neg = dti < 0, big = (dti >> 52) != 0;
+            uint64_t sc = 0;
+            if (!lost) {
                 for (int r = r_lo; r <= r_hi; ++r) {
-                    const int64_t cv = int64_t(rawc[col(r)]), xv = int64_t(rawx[col(r)]);
-                    neg |= (cv < 0) | (xv < 0);
-                    big |= ((cv | xv) >> 52) != 0;
+                    const int64_t cv = int64_t(raw[col(r)]);
+                    neg |= cv < 0;
+                    big |= (cv >> 52) != 0;
                     sc += uint64_t(cv);
+                }
+                uint64_t oc = warp_excl_scan_u64(sc, lane);
+                for (int r = r_lo; r <= r_hi; ++r) {
+                    oc += raw[col(r)];
+                    urow[r] = int32_t(oc);
+                }
+                sc = warp_sum_u64(sc);
+                __syncwarp();  // every lane has read the row before the next one lands
+                lost = stage(a.xfer + i * L);
+            }
+            uint64_t cx_lane = 0;
+            if (!lost) {
+                for (int r = r_lo; r <= r_hi; ++r) {
+                    const int64_t xv = int64_t(raw[col(r)]);
+                    neg |= xv < 0;
+                    big |= (xv >> 52) != 0;
                     sx += uint64_t(xv);
+                    cx_lane += uint64_t(xv) < sc ? uint64_t(xv) : sc;
                 }
                 neg = __any_sync(0xffffffffu, neg);
                 big = __any_sync(0xffffffffu, big);
-                sc = warp_sum_u64(sc);
                 sx = warp_sum_u64(sx);
+            }
+            if (lost) {
+                if (lane == 0) {
+                    a.makespan[i] = -int64_t(DC_ERR_INTERNAL);
+                    if (a.nseg) a.nseg[i] = 0;
+                    if (a.status) a.status[i] = DC_ERR_INTERNAL;
+                }
+                for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
+                flag = lost == 1 ? int(kListed) : int(kAbort);
+            } else {
                 int st = DC_OK;
                 if (neg)
                     st = DC_ERR_NEGATIVE;
@@ -467,15 +490,8 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
                     for (int w = lane; w < W; w += 32) a.bits[i * W + w] = 0u;
                     flag = kListed;  // done: nothing for the other warps
                 } else {
-                    // capped transfers; the arithmetic form
-                    uint64_t cx = 0, cc = 0;
-                    for (int r = r_lo; r <= r_hi; ++r) {
-                        const uint64_t xv = rawx[col(r)];
-                        cx += xv < sc ? xv : sc;
-                        cc += rawc[col(r)];
-                    }
-                    const uint64_t cx_lane = cx, cc_lane = cc;
-                    cx = warp_sum_u64(cx);
+                    // transfers capped at the total compute; the arithmetic form
+                    const uint64_t cx = warp_sum_u64(cx_lane);
                     shift = sx - cx;
                     const uint64_t bound = sc + cx + uint64_t(L) * uint64_t(dti);
                     if (bound <= kShiftedLimit)
@@ -492,15 +508,11 @@ __global__ void __launch_bounds__(32 * NW, NW == 1 ? 16 : 24 / NW) deep_kernel(D
                             if (DC_CHECK(int64_t(at) < a.lo + a.count)) a.list[at] = uint32_t(i);
                         }
                     } else {
-                        // prefix sums in processing order: comp (below 2^31) into
-                        // urow, capped transfers (64-bit) into the slot
-                        uint64_t oc = warp_excl_scan_u64(cc_lane, lane);
+                        // prefix of the capped transfers (64-bit) into the slot
                         uint64_t ox = warp_excl_scan_u64(cx_lane, lane);
                         for (int r = r_lo; r <= r_hi; ++r) {
-                            const uint64_t xv = rawx[col(r)];
-                            oc += rawc[col(r)];
+                            const uint64_t xv = raw[col(r)];
                             ox += xv < sc ? xv : sc;
-                            urow[r] = int32_t(oc);
                             P64[r] = ox;
                         }
                         if (lane == 0) {
