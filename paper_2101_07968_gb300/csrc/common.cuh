@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cstdlib>
 #include <mutex>
 
 #include <cuda_runtime.h>
@@ -145,6 +146,18 @@ struct NvtxRange {
     NvtxRange(const NvtxRange &) = delete;
     NvtxRange &operator=(const NvtxRange &) = delete;
 };
+
+// Test hook for the barrier discipline: DC_BLOCK_WARPS=1|2|4|8 in the
+// environment makes the looped, deep-chain and CTA-per-instance kernels run with
+// that many warps per CTA where the kernel allows it (results must not change);
+// unset or any other value keeps each kernel's own choice. Read on every launch.
+inline int forced_warps()
+{
+    const char *e = std::getenv("DC_BLOCK_WARPS");
+    if (!e) return 0;
+    const int v = std::atoi(e);
+    return (v == 1 || v == 2 || v == 4 || v == 8) ? v : 0;
+}
 
 // A per-device launch fact (resident CTAs per SM of a kernel, the SM count),
 // found once per device by the first call that needs it; `lookup` may also

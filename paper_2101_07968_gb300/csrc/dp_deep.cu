@@ -820,6 +820,12 @@ cudaError_t launch_deep_dir(const DeepArgs &a, int64_t nslots, bool pdl, cudaStr
             grid_pick = G;
         }
     }
+    if (const int f = forced_warps()) {  // the test hook's warps per instance
+        pick = f == 1 ? 0 : f == 2 ? 1 : f == 4 ? 2 : 3;
+        grid_pick = int64_t(nb[pick]) * sms;
+        if (grid_pick > nslots) grid_pick = nslots;
+        if (grid_pick > a.count) grid_pick = a.count;
+    }
     switch (nws[pick]) {
         case 1: return launch_deep_nw<FWD, 1>(a, grid_pick, pdl, stream);
         case 2: return launch_deep_nw<FWD, 2>(a, grid_pick, pdl, stream);

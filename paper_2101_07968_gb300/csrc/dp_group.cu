@@ -984,7 +984,7 @@ cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp
     GroupArgs a{batch, L, comp, xfer, dt, makespan, bits, nseg, status, list_count, list,
                 static_cast<unsigned char *>(tables)};
     const size_t smem = group_smem_bytes(L, tables == nullptr);
-    const int nt = group_threads(L);
+    const int nt = forced_warps() ? 32 * forced_warps() : group_threads(L);
     cudaError_t e;
     if (forward) {
         e = cudaFuncSetAttribute(group_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -496,7 +496,12 @@ cudaError_t launch_mid(bool forward, int64_t batch, int L, const int64_t *comp,
                                              status, ticket, list_count, list, tb, stream)       \
                    : launch_mid_nw<false, NW>(batch, L, comp, xfer, dt, makespan, bits, nseg,   \
                                               status, ticket, list_count, list, tb, stream);
-    switch (mid_warps(L)) {
+    // warps per tile: the kernel's choice, or the test hook's when its blocks
+    // (4 per warp and column) still cover a column's rows
+    int nw = mid_warps(L);
+    const int f = forced_warps();
+    if (f == 1 || (f > 1 && (L + 6) / 8 <= 4 * f)) nw = f;
+    switch (nw) {
         case 1: DC_MID_LAUNCH(1)
         case 2: DC_MID_LAUNCH(2)
         case 4: DC_MID_LAUNCH(4)
