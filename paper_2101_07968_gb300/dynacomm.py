@@ -358,9 +358,13 @@ class StepGraph:
     """One whole step for a fixed config -- dc_profile_gen, the forward and backward
     DPs and the f_m replay of both decisions -- captured once as a CUDA graph and
     replayed. For small batches the host cost of the step's launches exceeds the
-    kernels' own time; replay() issues them as one graph launch. After each
-    replay(): prof (fc, pt, bc, gt, dt), sched.out[d] and replay_out[d] for d in
-    (FWD, BWD) hold that step's results."""
+    kernels' own time; replay() issues them as one graph launch. The two
+    directions are independent, so after the generator they run on two branches
+    of the graph (each with its own workspace): one direction's kernels start on
+    the SMs the other's tail leaves free, and a replay kernel (memory-bound) can
+    run beside the other direction's DP (integer-ALU-bound). After each replay():
+    prof (fc, pt, bc, gt, dt), sched.out[d] and replay_out[d] for d in (FWD, BWD)
+    hold that step's results."""
 
     def __init__(self, cfg: dict, device="cuda"):
         import torch
@@ -372,8 +376,11 @@ class StepGraph:
                      for k in ("fc", "pt", "bc", "gt")}
         self.prof["dt"] = torch.empty(B, dtype=torch.int64, device=device)
         self.sched = Scheduler(B, L, device=device)
+        self.sched_b = Scheduler(B, L, device=device)  # the backward branch's workspace
+        self.sched.out[BWD] = self.sched_b.out[BWD]
         self.replay_out = {d: torch.empty(B, dtype=torch.int64, device=device)
                            for d in (FWD, BWD)}
+        self._branch = torch.cuda.Stream(device=device)
         # one eager step first: one-time setup (function attributes, occupancy
         # queries) happens outside the capture
         side = torch.cuda.Stream(device=device)
@@ -386,14 +393,24 @@ class StepGraph:
         with torch.cuda.graph(self.graph):
             self._step()
 
+    def _direction(self, d, sched):
+        p = self.prof
+        c, x = ("fc", "pt") if d == FWD else ("bc", "gt")
+        o = sched.run(d, p[c], p[x], p["dt"])
+        _check(dc_eval_timeline_batch(self.B, self.L, d, p[c], p[x], p["dt"], o["bits"],
+                                      self.replay_out[d]), "dc_eval_timeline_batch")
+
     def _step(self):
+        import torch
         p = self.prof
         _check(dc_profile_gen(self.c, p["fc"], p["pt"], p["bc"], p["gt"], p["dt"]),
                "dc_profile_gen")
-        for d, (c, x) in ((FWD, ("fc", "pt")), (BWD, ("bc", "gt"))):
-            o = self.sched.run(d, p[c], p[x], p["dt"])
-            _check(dc_eval_timeline_batch(self.B, self.L, d, p[c], p[x], p["dt"], o["bits"],
-                                          self.replay_out[d]), "dc_eval_timeline_batch")
+        main = torch.cuda.current_stream()
+        self._branch.wait_stream(main)  # the backward branch starts after the generator
+        self._direction(FWD, self.sched)
+        with torch.cuda.stream(self._branch):
+            self._direction(BWD, self.sched_b)
+        main.wait_stream(self._branch)
 
     def replay(self):
         self.graph.replay()

@@ -1,5 +1,6 @@
-"""A whole step captured as a CUDA graph (dynacomm.StepGraph) gives, replay after
-replay, exactly the eager path's profiles, decisions, makespans and replays."""
+"""A whole step captured as a CUDA graph (dynacomm.StepGraph, the two directions on
+parallel branches with their own workspaces) gives, replay after replay, exactly
+the eager path's profiles, decisions, makespans and replays."""
 import pytest
 
 from paper_2101_07968_gb300 import workloads as wl
@@ -19,7 +20,7 @@ def dc():
 
 
 @pytest.mark.parametrize("name,batch", [("tiny", 4096), ("vgg16", 20_011), ("resnet50", 3_001),
-                                        ("alexnet", 1)])
+                                        ("alexnet", 1), ("deepchain", 300)])
 def test_step_graph_equals_eager(dc, name, batch):
     import torch
     cfg = wl.with_batch(wl.config(name), batch, inst0=7)
