@@ -50,7 +50,7 @@ __device__ __forceinline__ void fused_direction(const GenParams &g, const GenTab
                                                 int64_t *stX, int32_t *lw, int lane,
                                                 const FusedOut &o)
 {
-    using K = Small<L, uint32_t, kKeepCols>;
+    using K = Tab32<L>;
     constexpr int W = (L - 1 + 31) / 32;
     constexpr int dir = FWD ? 0 : 1;
     __syncwarp();  // every lane is done with the area (the table of the other direction)
@@ -85,7 +85,7 @@ template <int L, bool FWD>
 __global__ void __launch_bounds__(32, DC_SMALL_MINB)
     fused_dense_kernel(const __grid_constant__ GenParams g, const GenTables *t, const FusedOut o)
 {
-    using K = Small<L, uint32_t, kKeepCols>;
+    using K = Tab32<L>;
     extern __shared__ __align__(16) unsigned char smem[];
     const int lane = threadIdx.x;
     int64_t *stC = reinterpret_cast<int64_t *>(smem);
@@ -169,22 +169,21 @@ template <int L, bool FWD>
 cudaError_t launch_fused_dir(const GenParams &g, const GenTables *t, const FusedOut &o,
                              cudaStream_t stream)
 {
-    using K32 = Small<L, uint32_t, kKeepCols>;
     static DeviceCache resident;  // single-warp CTAs of the fused kernel per SM
     int per_sm = 0;
     cudaError_t le = resident.get(per_sm, [](int &n) {
         cudaError_t e = cudaFuncSetAttribute(fused_dense_kernel<L, FWD>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             K32::kWarpBytes);
+                                             Tab32<L>::kSharedBytes);
         if (e != cudaSuccess) return e;
         return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fused_dense_kernel<L, FWD>, 32,
-                                                             K32::kWarpBytes);
+                                                             Tab32<L>::kSharedBytes);
     });
     if (le != cudaSuccess) return le;
     const int64_t tiles = (g.batch + 31) / 32;
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;
-    fused_dense_kernel<L, FWD><<<unsigned(grid), 32, K32::kWarpBytes, stream>>>(g, t, o);
+    fused_dense_kernel<L, FWD><<<unsigned(grid), 32, Tab32<L>::kSharedBytes, stream>>>(g, t, o);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     return launch_fused_list<L, FWD>(g, t, o, stream);

@@ -18,12 +18,12 @@
 //    Path[m][n] as the lowest k whose candidate equals the cell, which is the k
 //    Algorithm 3/4 keeps with its strict-improvement test. A step compares all
 //    of its candidates at once (bit mask, lowest set bit), and every step runs
-//    the same code (column 1 is stored like the others), so the lanes of a warp
-//    at different depths do not split into separate paths. The pass stores only
-//    columns 1..kKeepCols: the traceback of an s-segment optimum reads columns
-//    1..s-1 only, and s is small in practice (2-5 on CNN-shaped profiles); an
-//    instance whose s needs a deeper column is re-solved by the 64-bit pass,
-//    which keeps every column;
+//    the same code (column 1 is read as U less a constant, the other kept
+//    columns from the table), so the lanes of a warp at different depths do not
+//    split into separate paths. The pass keeps only columns 1..kKeepCols: the
+//    traceback of an s-segment optimum reads columns 1..s-1 only, and s is small
+//    in practice (2-5 on CNN-shaped profiles); an instance whose s needs a
+//    deeper column is re-solved by the 64-bit pass, which keeps every column;
 //  * a row whose costs all fit 32 bits (compute below 2^31 / L) gets its prefix
 //    sums in 32-bit arithmetic (fast_uv); other rows take the 64-bit prefix,
 //    which also classifies bad input;
@@ -34,23 +34,43 @@
 //    that a 64-bit instantiation of the literal template solves afterwards; that
 //    pass is launched early and waits in hardware for this one (programmatic
 //    dependent launch);
-//  * persistent warps: each warp walks 32-instance tiles. A tile's rows arrive
-//    by cp.async (coalesced 16-byte copies of cost pairs for even L) in the
-//    warp's own table area, with a row stride at which every lane reads its own
-//    row without bank conflicts (stage_stride); the prefix sums then leave them
-//    in registers and the table overwrites them. Sharing the area keeps a warp
-//    at the table's size of shared memory, so 20 warps fit on an SM (the
-//    register limit at <= 96 registers): more resident warps hide more latency
-//    than a separate prefetch buffer would. Instead, while a tile is solved its
-//    successor is prefetched into L2, so that the next copies wait less.
+//  * persistent single-warp CTAs walk 32-instance tiles. A tile's rows arrive by
+//    cp.async (coalesced 16-byte copies of cost pairs for even L) at a row
+//    stride at which every lane reads its own row without bank conflicts
+//    (stage_stride); the prefix sums then leave them in registers. Short rows
+//    (L < kSplitMinL) stage in the warp's table area, which keeps a warp small
+//    (many resident warps) while the next tile is prefetched into L2; longer
+//    rows stage beside the table, so that the next tile's copies are in flight
+//    while this one is solved, and take their tiles from a ticket (see the
+//    kernel).
 #include "dp_small.cuh"
 
 namespace dc {
 namespace {
 
-// 32-bit pass over the whole batch; persistent warps, tiles staged in the table area.
+// From this L on the dense pass stages each tile beside the table and takes its
+// tiles from a ticket (the split design below); shorter rows share one area
+// and take every grid-th tile.
+constexpr int kSplitMinL = 12;
+
+// Resident single-warp CTAs per SM the registers must allow: the split design
+// is held to 12 by its shared memory, so its registers may grow to that.
+__host__ __device__ constexpr int dense_min_ctas(int L) { return L >= kSplitMinL ? 12 : DC_SMALL_MINB; }
+
+// 32-bit pass over the whole batch; persistent single-warp CTAs.
+//  * shared design (L < kSplitMinL): a tile's rows are staged in the warp's table
+//    area, so a warp holds only max(rows, table) of shared memory and many warps
+//    fit an SM; while a tile is solved its successor is prefetched into L2. Tiles
+//    are dealt statically (warp w takes w, w + grid, ...): short tiles, for which
+//    one atomic per tile on a shared ticket would cost more than the balance gains.
+//  * split design (L >= kSplitMinL): the staging lies beside the table, and the
+//    copies of the warp's next tile (rows and dt) are issued as soon as this
+//    tile's rows are read, so they land while it is solved. Tiles come from an
+//    atomic ticket, claimed one tile ahead: warps on a crowded sub-partition
+//    progress more slowly than others, and a static deal would leave the SMs
+//    emptying out behind the slowest warps.
 template <int L, bool FWD>
-__global__ void __launch_bounds__(32, DC_SMALL_MINB)
+__global__ void __launch_bounds__(32, dense_min_ctas(L))
     small_dense_kernel(int64_t batch, const int64_t *__restrict__ comp,
                        const int64_t *__restrict__ xfer, const int64_t *__restrict__ dt,
                        int64_t *__restrict__ makespan, uint32_t *__restrict__ bits,
@@ -58,44 +78,28 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
                        uint32_t *__restrict__ wide_count, uint32_t *__restrict__ wide_list,
                        bool pairs)
 {
-    using K = Small<L, uint32_t, kKeepCols>;
+    using K = Tab32<L>;
     constexpr int W = (L - 1 + 31) / 32;
+    constexpr bool kSplit = L >= kSplitMinL;
     extern __shared__ __align__(16) unsigned char smem[];
     const int lane = threadIdx.x;
-    int64_t *stC = reinterpret_cast<int64_t *>(smem);
-    int64_t *stX = stC + 32 * K::kStride;
     int32_t *lw = reinterpret_cast<int32_t *>(smem) + lane;
+    int64_t *stC = reinterpret_cast<int64_t *>(smem + (kSplit ? K::kBytes : 0));
+    int64_t *stX = stC + 32 * K::kStride;
+    int64_t *stD = stX + 32 * K::kStride;  // the tile's dt (split design)
+    uint32_t *ticket = wide_count + 1;     // tiles handed out (zero before the launch)
 
     const int64_t tiles = (batch + 31) / 32;
-    int64_t tile = blockIdx.x;
     pdl_trigger();  // the list pass may be scheduled as soon as CTAs of this one exit
-    if (tile >= tiles) return;
     auto rows_of = [&](int64_t t) { return int(batch - t * 32 < 32 ? batch - t * 32 : 32); };
-    for (; tile < tiles; tile += gridDim.x) {
-        const int64_t base = tile * 32;
-        const int rows = rows_of(tile);
-        __syncwarp();  // every lane is done with the table: stage the tile's rows there
-        stage_tile<L>(stC, stX, comp, xfer, base, rows, lane, pairs);
-        if (tile + gridDim.x < tiles) {  // the warp's next tile into L2, one 128-byte line per lane and array
-            const int64_t nbase = (tile + gridDim.x) * 32;
-            if (lane * 16 < rows_of(tile + gridDim.x) * L) {
-                asm volatile("prefetch.global.L2 [%0];" ::"l"(comp + nbase * L + lane * 16));
-                asm volatile("prefetch.global.L2 [%0];" ::"l"(xfer + nbase * L + lane * 16));
-            }
-        }
-        const int64_t i = base + lane;
-        const bool active = lane < rows;
-        const int64_t dti = active ? __ldg(dt + i) : 0;
-        cp_async_wait_all();
-        __syncwarp();
-        const int64_t *rc = stC + lane * K::kStride, *rx = stX + lane * K::kStride;
-        int32_t U[L + 1], V[L + 1];
-        uint64_t xraw;
-        bool wide;
-        int st;
-        row_uv<L, FWD>(rc, rx, dti, U, V, xraw, wide, st);
-        __syncwarp();  // rows read: the lanes' table slices may be written
-        if (!active) continue;
+    auto claim = [&]() {
+        uint32_t v = 0;
+        if (lane == 0) v = atomicAdd(ticket, 1u);
+        return v;
+    };
+    // the solve of one tile's rows, held by each lane in U, V
+    auto finish = [&](int64_t i, const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
+                      int64_t dti, uint64_t xraw, bool wide, int st) {
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
         } else if (wide ||
@@ -103,6 +107,69 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
             // 64-bit values, or a traceback deeper than the kept columns: work list
             const uint32_t at = atomicAdd(wide_count, 1u);
             if (DC_CHECK(int64_t(at) < batch)) wide_list[at] = uint32_t(i);
+        }
+    };
+
+    if constexpr (kSplit) {
+        auto stage = [&](int64_t t) {
+            const int64_t b = t * 32;
+            const int r = rows_of(t);
+            if (lane < r) cp_async8(stD + lane, dt + b + lane);
+            stage_tile<L>(stC, stX, comp, xfer, b, r, lane, pairs);  // commits the group
+        };
+        int64_t tile = int64_t(__shfl_sync(0xffffffffu, claim(), 0));
+        if (tile >= tiles) return;
+        stage(tile);
+        uint32_t next_raw = claim();  // claimed a tile ahead: its copies go out mid-tile
+        while (tile < tiles) {
+            const int64_t i = tile * 32 + lane;
+            const bool active = lane < rows_of(tile);
+            cp_async_wait_all();
+            __syncwarp();
+            const int64_t dti = active ? stD[lane] : 0;
+            int32_t U[L + 1], V[L + 1];
+            uint64_t xraw;
+            bool wide;
+            int st;
+            row_uv<L, FWD>(stC + lane * K::kStride, stX + lane * K::kStride, dti, U, V, xraw,
+                           wide, st);
+            __syncwarp();  // the staging is read: the next tile's copies may land there
+            const int64_t next = int64_t(__shfl_sync(0xffffffffu, next_raw, 0));
+            if (next < tiles) {
+                stage(next);
+                next_raw = claim();
+            }
+            tile = next;
+            if (active) finish(i, U, V, dti, xraw, wide, st);
+        }
+    } else {
+        int64_t tile = blockIdx.x;
+        if (tile >= tiles) return;
+        for (; tile < tiles; tile += gridDim.x) {
+            const int64_t base = tile * 32;
+            const int rows = rows_of(tile);
+            __syncwarp();  // every lane is done with the table: stage the tile's rows there
+            stage_tile<L>(stC, stX, comp, xfer, base, rows, lane, pairs);
+            if (tile + gridDim.x < tiles) {  // the warp's next tile into L2, one 128-byte line per lane and array
+                const int64_t nbase = (tile + gridDim.x) * 32;
+                if (lane * 16 < rows_of(tile + gridDim.x) * L) {
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(comp + nbase * L + lane * 16));
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(xfer + nbase * L + lane * 16));
+                }
+            }
+            const int64_t i = base + lane;
+            const bool active = lane < rows;
+            const int64_t dti = active ? __ldg(dt + i) : 0;
+            cp_async_wait_all();
+            __syncwarp();
+            int32_t U[L + 1], V[L + 1];
+            uint64_t xraw;
+            bool wide;
+            int st;
+            row_uv<L, FWD>(stC + lane * K::kStride, stX + lane * K::kStride, dti, U, V, xraw,
+                           wide, st);
+            __syncwarp();  // rows read: the lanes' table slices may be written
+            if (active) finish(i, U, V, dti, xraw, wide, st);
         }
     }
 }
@@ -163,26 +230,25 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
                        int32_t *status, uint32_t *wide_count, uint32_t *wide_list,
                        cudaStream_t stream)
 {
-    using K32 = Small<L, uint32_t, kKeepCols>;
     using K64 = Small<L, uint64_t, L>;
+    constexpr int kSmem = L >= kSplitMinL ? Tab32<L>::kSplitBytes : Tab32<L>::kSharedBytes;
     static DeviceCache resident;  // single-warp CTAs of the dense kernel per SM
     int per_sm = 0;
     cudaError_t le = resident.get(per_sm, [](int &n) {
         cudaError_t e = cudaFuncSetAttribute(small_dense_kernel<L, FWD>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             K32::kWarpBytes);
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
         if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(small_list_kernel<L, FWD>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, K64::kTableBytes);
         if (e != cudaSuccess) return e;
         return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, small_dense_kernel<L, FWD>, 32,
-                                                             K32::kWarpBytes);
+                                                             kSmem);
     });
     if (le != cudaSuccess) return le;
     const int64_t tiles = (batch + 31) / 32;
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;
-    small_dense_kernel<L, FWD><<<unsigned(grid), 32, K32::kWarpBytes, stream>>>(
+    small_dense_kernel<L, FWD><<<unsigned(grid), 32, kSmem, stream>>>(
         batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list,
         ((reinterpret_cast<uintptr_t>(comp) | reinterpret_cast<uintptr_t>(xfer)) & 15u) == 0);
     cudaError_t e = cudaGetLastError();

@@ -40,20 +40,36 @@ __host__ __device__ constexpr int stage_stride(int L)
     return (L % 2 == 1) ? L : (L % 4 == 2 ? L : L + 2);
 }
 
-// Stored columns 2..C with C = min(keep, L-1); KEEP = L keeps them all.
+// Table of the 64-bit pass: stored columns 2..C with C = min(keep, L-1) (KEEP = L
+// keeps them all), then S[0..L] and R[0..L].
 template <int L, typename T, int KEEP>
 struct Small {
     static constexpr int kLast = KEEP < L - 1 ? KEEP : L - 1;  // last stored column
     static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
-    static constexpr int kOffS = kCells;   // S[0..L] (64-bit pass)
-    static constexpr int kOffC1 = kCells;  // column 1, rows 1..L-1 (32-bit pass)
-    static constexpr int kOffR = kCells + L + 1;                        // R[0..L]
+    static constexpr int kOffS = kCells;          // S[0..L]
+    static constexpr int kOffR = kCells + L + 1;  // R[0..L]
     static constexpr int kLaneVals = kCells + 2 * (L + 1);
-    static constexpr int kStride = stage_stride(L);          // staging row stride (int64, odd)
-    static constexpr int kStageBytes = 2 * 32 * kStride * 8;   // comp + xfer rows of a tile
     static constexpr int kTableBytes = 32 * kLaneVals * int(sizeof(T));
-    // staging and table share the warp's area
-    static constexpr int kWarpBytes = kStageBytes > kTableBytes ? kStageBytes : kTableBytes;
+};
+
+// Shared memory of a warp of the 32-bit pass. Its table, per lane (32-bit words,
+// lane-interleaved): word 0 unused, the kept cells of columns 2..kLast at
+// 1 + cell2 (a traceback step loads one word below a column's first cell, which
+// stays inside the table), then U[0..L]; column 1 is not stored, being U shifted
+// by a constant. The tile's staging (comp and xfer rows at a padded stride, then
+// dt) either shares the table's area (kSharedBytes) or lies beside it
+// (kSplitBytes), so that the next tile can land while this one is solved.
+template <int L>
+struct Tab32 {
+    static constexpr int kLast = kKeepCols < L - 1 ? kKeepCols : L - 1;  // last stored column
+    static constexpr int kCells = kLast >= 2 ? cell2(L, L, kLast) + 1 : 0;
+    static constexpr int kOffU = 1 + kCells;
+    static constexpr int kWords = kOffU + L + 1;
+    static constexpr int kBytes = 32 * kWords * 4;
+    static constexpr int kStride = stage_stride(L);               // staging row stride (int64)
+    static constexpr int kRowsBytes = 2 * 32 * kStride * 8;        // comp + xfer rows of a tile
+    static constexpr int kSharedBytes = kRowsBytes > kBytes ? kRowsBytes : kBytes;
+    static constexpr int kSplitBytes = kBytes + kRowsBytes + 32 * 8;  // table | rows | dt
 };
 
 template <typename T>
@@ -237,15 +253,12 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
                                        int32_t dt, int32_t fcL, int32_t *lw, int32_t &bestV,
                                        int &best_s)
 {
-    using K = Small<L, uint32_t, kKeepCols>;
+    using K = Tab32<L>;
     // forward: U = Q, V = G, col = A; backward: U = BC - dt, V = NGT, col = F
     const int32_t dt2 = 2 * dt;
     int32_t col[L + 1];
 #pragma unroll
-    for (int m = 1; m <= L; ++m) {
-        col[m] = FWD ? fcL + U[m] - dt : U[m] + dt;
-        if (m < L) lw[32 * (K::kOffC1 + m)] = col[m];  // for the traceback
-    }
+    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL + U[m] - dt : U[m] + dt;
     bestV = FWD ? fcL + dt : U[L] + dt2;
     best_s = 1;
 #pragma unroll
@@ -261,7 +274,7 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
             const int32_t b = min_fold3<L>(c, cnt);
             if (m == L) last = FWD ? b - U[L] : b;
             col[m] = FWD ? b - dt : b + dt;
-            if (n <= K::kLast) lw[32 * cell2(L, m, n)] = col[m];
+            if (n <= K::kLast) lw[32 * (1 + cell2(L, m, n))] = col[m];
         }
         const int32_t v = FWD ? last + n * dt : last + dt2;  // X[L][n] - P[L] or X[L][n] - S[L]
         if (v < bestV) {  // strict: the lowest n wins ties
@@ -282,11 +295,11 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
                                          int64_t *makespan, uint32_t *bits, int32_t *nseg,
                                          int32_t *status)
 {
-    using K = Small<L, uint32_t, kKeepCols>;
+    using K = Tab32<L>;
     constexpr int W = (L - 1 + 31) / 32;
     const int32_t fcL = V[0];  // forward: FC[L]
 #pragma unroll
-    for (int m = 0; m <= L; ++m) lw[32 * (K::kOffR + m)] = U[m];  // the traceback reads U[m]
+    for (int m = 0; m <= L; ++m) lw[32 * (K::kOffU + m)] = U[m];  // the traceback reads U[m]
     int32_t bestV;
     int s;
     fill_e<L, FWD>(U, V, dt, fcL, lw, bestV, s);
@@ -294,23 +307,29 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
 
     // from (L, s) step to the lowest k whose candidate equals the cell, set
     // p_k / g_k, continue at (k, n-1). A step compares every candidate at once
-    // (U and V still in registers, compile-time k): bit k of `hit` is set when
+    // (V still in registers, compile-time k): bit k of `hit` is set when
     // candidate k equals the cell, and the lowest k inside [n-1, m-1] is the one
-    // Algorithm 3/4 keeps.
+    // Algorithm 3/4 keeps. The loads of k outside that range read other words of
+    // the lane's table and are masked off.
     uint32_t word = 0;
     int err = 0;
     int m = L, n = s;
     int32_t target = FWD ? bestV - s * dt + U[L] : bestV - 2 * dt;  // B[L][s] + Q[L] or F[L][s] - dt
+    // column 1 is U shifted by off1 (A[k][1] = FC[L] + U[k] - dt forward, F[k][1] =
+    // U[k] + dt backward): its step reads U and compares the candidate and the
+    // cell both less off1, max(u + V, f + off1) = max(u - off1 + V, f) + off1
+    const int32_t off1 = FWD ? fcL - dt : dt;
     while (n > 1) {
         const int nm1 = n - 1;
-        const int32_t u = lds(lw, K::kOffR + m);
-        // cell (k, n-1) is base + k; column 1 has its own row of the table
-        const int base = nm1 == 1 ? K::kOffC1 : cell2(L, 0, nm1);
+        const int32_t off = nm1 == 1 ? off1 : 0;
+        const int32_t u = lds(lw, K::kOffU + m) - off;
+        const int32_t tgt = target - off;
+        // cell (k, n-1) of a kept column is word base + k (>= 0 for every k >= 1)
+        const int base = nm1 == 1 ? K::kOffU : 1 + cell2(L, 0, nm1);
         uint32_t hit = 0u;
 #pragma unroll
         for (int k = 1; k < L; ++k) {
-            const int32_t f = k >= nm1 ? lds(lw, base + k) : 0;
-            if (__viaddmax_s32(u, V[k], f) == target) hit |= 1u << k;
+            if (__viaddmax_s32(u, V[k], lds(lw, base + k)) == tgt) hit |= 1u << k;
         }
         hit &= ((2u << (m - 1)) - 1u) & ~((1u << nm1) - 1u);  // k in [n-1, m-1]
         if (hit == 0u) {  // cannot happen: the fill and this check use the same arithmetic
@@ -319,7 +338,7 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
         }
         const int k = __ffs(int(hit)) - 1;
         word |= 1u << ((k - 1) & 31);
-        const int32_t fk = lds(lw, base + k);  // the cell (k, n-1): B + Q[k] = A + dt, or F - dt
+        const int32_t fk = lds(lw, base + k) + off;  // the cell (k, n-1): B + Q[k] = A + dt, or F - dt
         target = FWD ? fk + dt : fk - dt;
         m = k;
         n = nm1;

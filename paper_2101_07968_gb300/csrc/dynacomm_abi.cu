@@ -17,9 +17,10 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
 {
     unsigned char *ws = static_cast<unsigned char *>(workspace);
     if (L <= kSmallLMax) {
+        // header: work-list counter, then the dense pass's tile ticket
         uint32_t *count = reinterpret_cast<uint32_t *>(ws);
         uint32_t *list = reinterpret_cast<uint32_t *>(ws + 256);
-        cudaError_t e = cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
+        cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(uint32_t), stream);
         if (e != cudaSuccess) return e;
         // 32-bit pass over the batch, then a 64-bit pass over the instances it listed
         return launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
