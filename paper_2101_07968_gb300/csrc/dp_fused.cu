@@ -12,8 +12,8 @@ namespace {
 // into its row of the staging area, then the tile is solved as in dp_small.cu;
 // one pass per direction, each with its own list pass, which regenerates the
 // listed instances' rows.
-// workspace: [0, 256) the two list counters, [256, 256 + 8 batch) the two lists,
-// then the generator's tables
+// workspace: [0, 256) the two list counters and the two tile tickets,
+// [256, 256 + 8 batch) the two lists, then the generator's tables
 inline size_t fused_tables_offset(int64_t batch) { return (256 + 8 * size_t(batch) + 255) / 256 * 256; }
 
 struct FusedOut {
@@ -21,6 +21,7 @@ struct FusedOut {
     uint32_t *bits[2];
     int32_t *nseg[2], *status[2];
     uint32_t *wide_count[2], *wide_list[2];
+    uint32_t *ticket[2];  // tiles handed out per direction (zero before the launches)
 };
 
 // The generator's lookup tables, copied once per call from the parameter block
@@ -92,16 +93,32 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
     int64_t *stX = stC + 32 * K::kStride;
     int32_t *lw = reinterpret_cast<int32_t *>(smem) + lane;
     const int64_t tiles = (g.batch + 31) / 32;
-    int64_t tile = blockIdx.x;
     pdl_trigger();
-    if (tile >= tiles) return;
-    for (; tile < tiles; tile += gridDim.x) {
+    auto solve_tile = [&](int64_t tile) {
         const int64_t i = tile * 32 + lane;
         const bool active = i < g.batch;
         const int64_t gi = g.inst0 + i;
         InstanceDraws d = {};
         if (active) d = instance_draws(g, t->rate, t->bw, gi);
         fused_direction<L, FWD>(g, t, d, gi, i, active, stC, stX, lw, lane, o);
+    };
+    if constexpr (L >= kSplitMinL) {
+        // tiles from a ticket, the next claimed while this one is solved (as in
+        // the dense pass: warps sharing a sub-partition progress at different rates)
+        uint32_t *ticket = o.ticket[FWD ? 0 : 1];
+        auto claim = [&]() {
+            uint32_t v = 0;
+            if (lane == 0) v = atomicAdd(ticket, 1u);
+            return v;
+        };
+        int64_t tile = int64_t(__shfl_sync(0xffffffffu, claim(), 0));
+        while (tile < tiles) {
+            const uint32_t next_raw = claim();
+            solve_tile(tile);
+            tile = int64_t(__shfl_sync(0xffffffffu, next_raw, 0));
+        }
+    } else {
+        for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) solve_tile(tile);
     }
 }
 
@@ -217,8 +234,9 @@ cudaError_t launch_fused(const GenParams &g, int64_t *makespan, uint32_t *bits, 
         o.status[d] = status ? status + d * B : nullptr;
         o.wide_count[d] = reinterpret_cast<uint32_t *>(ws) + d;
         o.wide_list[d] = reinterpret_cast<uint32_t *>(ws + 256) + d * B;
+        o.ticket[d] = reinterpret_cast<uint32_t *>(ws) + 2 + d;
     }
-    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), stream);
+    cudaError_t e = cudaMemsetAsync(ws, 0, 4 * sizeof(uint32_t), stream);
     if (e != cudaSuccess) return e;
     GenTables *t = reinterpret_cast<GenTables *>(ws + fused_tables_offset(B));
     copy_tables_kernel<<<1, 256, 0, stream>>>(g, t);

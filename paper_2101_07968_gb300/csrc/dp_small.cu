@@ -48,11 +48,6 @@
 namespace dc {
 namespace {
 
-// From this L on the dense pass stages each tile beside the table and takes its
-// tiles from a ticket (the split design below); shorter rows share one area
-// and take every grid-th tile.
-constexpr int kSplitMinL = 12;
-
 // Resident single-warp CTAs per SM the registers must allow: the split design
 // is held to 12 by its shared memory, so its registers may grow to that.
 __host__ __device__ constexpr int dense_min_ctas(int L) { return L >= kSplitMinL ? 12 : DC_SMALL_MINB; }

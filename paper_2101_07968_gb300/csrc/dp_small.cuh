@@ -22,6 +22,11 @@ namespace {
 #define DC_TREE_MIN 1
 #endif
 constexpr int kTbGroup = 4;  // traceback candidates loaded per round
+// From this L on the dense and fused passes take their tiles from an atomic
+// ticket (and the dense pass stages each tile beside its table); shorter rows
+// take every grid-th tile, for which one atomic per tile costs more than the
+// balance gains.
+constexpr int kSplitMinL = 12;
 constexpr int kKeepCols = DC_KEEP_COLS;  // the 32-bit pass stores columns 2..kKeepCols
 
 // index of stored cell (m, n), 2 <= n <= L-1, n <= m <= L
