@@ -56,7 +56,9 @@ __device__ __forceinline__ void fused_direction(const GenParams &g, const GenTab
     constexpr int dir = FWD ? 0 : 1;
     __syncwarp();  // every lane is done with the area (the table of the other direction)
     if (active) {
-#pragma unroll
+        // rolled from kSplitMinL on: unrolled, the generator's divisions and the
+        // DP overflow the instruction cache (no_instruction leads the stalls)
+#pragma unroll (L >= kSplitMinL ? 1 : L)
         for (int l = 0; l < L; ++l) {
             int64_t params, flops, f, b, x;
             layer_draws(g, t->l0, t->l1, gi, l, params, flops);
