@@ -141,6 +141,13 @@ def dp_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+def first_pass_kernel(L: int) -> str:
+    """The kernel of a direction's first pass over the batch."""
+    if L <= 16:
+        return "small_dense_kernel"
+    return "mid_kernel" if L <= 256 else "deep_kernel"
+
+
 def binding_roof(*roofs, **extra):
     """The roof that binds: the one with the larger minimal time at peak, i.e. the
     larger achieved fraction; the others follow under other_roof (one) or
@@ -516,16 +523,20 @@ def run_ours(args):
         if world > 1:
             dist.barrier()
 
-    def step(ev=None):
+    def step(ev=None, kev=None):
         if ev is not None:
             ev[0].record()
         assert dc.dc_profile_gen(ccfg, prof["fc"], prof["pt"], prof["bc"], prof["gt"],
                                  prof["dt"]) == 0
         if ev is not None:
             ev[1].record()
+        if kev is not None:  # the library records kev[0..1] around the first pass's launches
+            assert dc.dc_time_next_pass(kev[0], kev[1]) == 0
         fo = sched.run(0, prof["fc"], prof["pt"], prof["dt"])
         if ev is not None:
             ev[2].record()
+        if kev is not None:
+            assert dc.dc_time_next_pass(kev[2], kev[3]) == 0
         bo = sched.run(1, prof["bc"], prof["gt"], prof["dt"])
         if ev is not None:
             ev[3].record()
@@ -561,6 +572,12 @@ def run_ours(args):
             sg, graph_error = None, f"{type(exc).__name__}: {exc}"
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    # the first pass of each direction, timed by the library on its stream
+    kevs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    for kv in kevs:
+        for e in kv:
+            e.record()  # creates the CUDA event the library will record
+    torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index if rank == 0 else -1) if rank == 0 else _Null() as clk:
@@ -582,6 +599,22 @@ def run_ours(args):
     eager_ms = max_over_ranks(start.elapsed_time(end) / max(args.steps, 1), dev)
     seg = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])
     gen_ms, fwd_ms, bwd_ms, eval_ms = seg.mean(axis=0)
+    # the first passes timed on their own launches, in K more eager steps (the
+    # events the library records between a first pass and its work-list pass
+    # stop the latter from being scheduled early, so they stay out of the steps
+    # timed above)
+    for s in range(args.steps):
+        step(None, kevs[s])
+    torch.cuda.synchronize()
+    kseg = np.array([[k[0].elapsed_time(k[1]), k[2].elapsed_time(k[3])] for k in kevs])
+    fwd_k_ms, bwd_k_ms = kseg.mean(axis=0)
+    # instances each direction's first pass left to its work-list pass (the same
+    # every step: the generator redraws the same batch)
+    listed = []
+    for d, (c, x) in ((0, ("fc", "pt")), (1, ("bc", "gt"))):
+        sched.run(d, prof[c], prof[x], prof["dt"])
+        torch.cuda.synchronize()
+        listed.append(int(sched.workspace[:4].view(torch.int32).item()))
     graph_ms = (max_over_ranks(g0.elapsed_time(g1) / max(args.steps, 1), dev)
                 if sg is not None else None)
     ms = graph_ms if graph_ms is not None else eager_ms
@@ -625,7 +658,12 @@ def run_ours(args):
     value = total / (ms * 1e-3)
     trans = 2 * transitions(L) * B
     dp_s = (fwd_ms + bwd_ms) * 1e-3
-    achieved = trans / dp_s / 1e9
+    # the dominant kernel: the first pass of both directions, timed on its own
+    # launches; its work is the instances it solved (the listed ones are left
+    # to the work-list pass)
+    first_s = (fwd_k_ms + bwd_k_ms) * 1e-3
+    first_trans = transitions(L) * (2 * B - listed[0] - listed[1])
+    achieved = first_trans / first_s / 1e9
     # ALU roof from unit counts: 4 x 16 integer-ALU lanes per SM per clock, the
     # 32-bit passes spend 1.5 ALU instructions per transition
     peak = sms * 64 * MAX_SM_MHZ * 1e6 / ALU_OPS_PER_TRANSITION / 1e9
@@ -634,7 +672,7 @@ def run_ours(args):
     if tr and tr.get("workload") == args.workload and tr.get("source_hash") == dp_source_hash():
         traffic = tr.get("bytes_per_launch")
     hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
-    dp_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
+    dp_gbs = dp_bytes(L) * (2 * B - listed[0] - listed[1]) / first_s / 1e9
     # kernels of this library per step: the generator; per direction the first
     # pass (split into several launches for long deep-chain batches) and the
     # pass over its work list; the two timeline replays
@@ -653,8 +691,20 @@ def run_ours(args):
                 "frac": dp_gbs / hbm_peak,
                 "bytes_per_instance_direction": dp_bytes(L),
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)"}
-    roofline = binding_roof(alu_roof, hbm_roof, kernel="dp_schedule (forward + backward)",
-                            traffic=traffic)
+    # the whole library call per direction (counter reset, first pass, work-list
+    # pass), against the same roofs
+    call_gtps = trans / dp_s / 1e9
+    call_gbs = 2 * dp_bytes(L) * B / dp_s / 1e9
+    dp_call = {"ms_forward": fwd_ms, "ms_backward": bwd_ms,
+               "alu_frac": call_gtps / peak, "hbm_frac": call_gbs / hbm_peak,
+               "note": "the whole dc_schedule_* call per direction: counter reset, "
+                       "first pass and work-list pass, all instances"}
+    roofline = binding_roof(alu_roof, hbm_roof,
+                            kernel=("first DP pass, forward + backward "
+                                    f"({first_pass_kernel(L)}), timed on its own launches"),
+                            kernel_ms={"forward": fwd_k_ms, "backward": bwd_k_ms},
+                            listed_to_work_list={"forward": listed[0], "backward": listed[1]},
+                            traffic=traffic, dp_call=dp_call)
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,

@@ -259,6 +259,22 @@ dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_t L, const 
 const char *dc_status_string(dc_status s);
 
 /* ------------------------------------------------------------------------
+ * dc_time_next_pass -- measurement support, not part of the method. The next
+ * dc_schedule_forward_batch, dc_schedule_backward_batch or
+ * dc_schedule_batch_static call made by the calling thread records `start` on
+ * its stream right before it launches its first pass over the batch (the
+ * dense, looped or deep-chain kernel, all of that pass's launches) and `stop`
+ * right after them, before its work-list pass; cudaEventElapsedTime(start,
+ * stop) is then that pass's time on the GPU. start, stop: events created by
+ * the caller on the current device, both non-NULL (DC_ERR_NULL if only one
+ * is); both NULL withdraw a pending request. The request belongs to the
+ * calling thread and is used up by its next schedule call, whether that call
+ * succeeds or not; no other call consumes it. This is the one state the
+ * library keeps between calls.
+ * ---------------------------------------------------------------------- */
+dc_status dc_time_next_pass(cudaEvent_t start, cudaEvent_t stop);
+
+/* ------------------------------------------------------------------------
  * dc_roof_int_probe -- measurement support, not part of the method: a
  * register-only loop of the DP's per-transition integer operations on
  * `blocks` x `threads` threads, `iters` iterations of 8 transitions each.

@@ -217,6 +217,14 @@ __device__ __forceinline__ T dmax(T a, T b) { return a > b ? a : b; }
 template <typename T>
 __device__ __forceinline__ T dmin(T a, T b) { return a < b ? a : b; }
 
+// A timing request (dc_time_next_pass) for the next schedule call made on this
+// thread: events recorded on the call's stream right before and right after the
+// launches of its first pass over the batch.
+struct PassEvents {
+    cudaEvent_t start = nullptr, stop = nullptr;
+};
+PassEvents take_pass_events();  // this thread's request, cleared (dynacomm_abi.cu)
+
 // Kernel launchers implemented in the .cu files.
 cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *comp,
                             const int64_t *xfer, const int64_t *dt, int64_t *makespan,
@@ -225,7 +233,8 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
 cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp,
                          const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                          uint32_t *bits, int32_t *nseg, int32_t *status,
-                         uint32_t *wide_count, uint32_t *wide_list, cudaStream_t stream);
+                         uint32_t *wide_count, uint32_t *wide_list, const PassEvents &pe,
+                         cudaStream_t stream);
 cudaError_t launch_group(bool forward, int64_t batch, int L, const int64_t *comp,
                          const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                          uint32_t *bits, int32_t *nseg, int32_t *status,

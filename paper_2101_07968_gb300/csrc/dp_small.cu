@@ -223,7 +223,7 @@ template <int L, bool FWD>
 cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
                        const int64_t *dt, int64_t *makespan, uint32_t *bits, int32_t *nseg,
                        int32_t *status, uint32_t *wide_count, uint32_t *wide_list,
-                       cudaStream_t stream)
+                       const PassEvents &pe, cudaStream_t stream)
 {
     using K64 = Small<L, uint64_t, L>;
     constexpr int kSmem = L >= kSplitMinL ? Tab32<L>::kSplitBytes : Tab32<L>::kSharedBytes;
@@ -243,11 +243,19 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
     const int64_t tiles = (batch + 31) / 32;
     int64_t grid = int64_t(sm_count()) * per_sm;
     if (grid > tiles) grid = tiles;
+    if (pe.start) {
+        const cudaError_t re = cudaEventRecord(pe.start, stream);
+        if (re != cudaSuccess) return re;
+    }
     small_dense_kernel<L, FWD><<<unsigned(grid), 32, kSmem, stream>>>(
         batch, comp, xfer, dt, makespan, bits, nseg, status, wide_count, wide_list,
         ((reinterpret_cast<uintptr_t>(comp) | reinterpret_cast<uintptr_t>(xfer)) & 15u) == 0);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    if (pe.stop) {
+        e = cudaEventRecord(pe.stop, stream);
+        if (e != cudaSuccess) return e;
+    }
     // the list length is known on the device only: persistent warps (4 per SM)
     // walk it, and the surplus exits at once
     int64_t lgrid = (batch + 31) / 32;
@@ -274,14 +282,15 @@ cudaError_t launch_dir(int64_t batch, const int64_t *comp, const int64_t *xfer,
 cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp,
                          const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                          uint32_t *bits, int32_t *nseg, int32_t *status,
-                         uint32_t *wide_count, uint32_t *wide_list, cudaStream_t stream)
+                         uint32_t *wide_count, uint32_t *wide_list, const PassEvents &pe,
+                         cudaStream_t stream)
 {
 #define DC_SMALL_CASE(LL)                                                                     \
     case LL:                                                                                  \
         return forward ? launch_dir<LL, true>(batch, comp, xfer, dt, makespan, bits, nseg,   \
-                                              status, wide_count, wide_list, stream)         \
+                                              status, wide_count, wide_list, pe, stream)     \
                        : launch_dir<LL, false>(batch, comp, xfer, dt, makespan, bits, nseg,  \
-                                               status, wide_count, wide_list, stream);
+                                               status, wide_count, wide_list, pe, stream);
     switch (L) {
         DC_SMALL_CASE(1) DC_SMALL_CASE(2) DC_SMALL_CASE(3) DC_SMALL_CASE(4)
         DC_SMALL_CASE(5) DC_SMALL_CASE(6) DC_SMALL_CASE(7) DC_SMALL_CASE(8)

@@ -1,12 +1,24 @@
 // C ABI entry points (declared in include/dynacomm.h): host-side argument
 // checks, then kernel launches on the caller's stream. No allocation, no
-// synchronisation, no state kept between calls.
+// synchronisation, no state kept between calls (save the timing request of
+// dc_time_next_pass, which the thread's next schedule call uses up).
 #include "gen_device.cuh"
 
 namespace dc {
 
 cudaError_t launch_gen(const dc_profile_cfg *c, int64_t *fc, int64_t *pt, int64_t *bc,
                        int64_t *gt, int64_t *dt, cudaStream_t stream);
+
+namespace {
+thread_local PassEvents t_pass_events;  // dc_time_next_pass's request for this thread
+}  // namespace
+
+PassEvents take_pass_events()
+{
+    const PassEvents pe = t_pass_events;
+    t_pass_events = PassEvents{};
+    return pe;
+}
 
 // Forward and backward solves share one path after the layers are put in
 // processing order (done inside the kernels).
@@ -16,6 +28,9 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
                             cudaStream_t stream)
 {
     unsigned char *ws = static_cast<unsigned char *>(workspace);
+    const PassEvents pe = take_pass_events();
+    // events around the first pass of a looped or deep-chain solve
+    auto mark = [&](cudaEvent_t ev) { return ev ? cudaEventRecord(ev, stream) : cudaSuccess; };
     if (L <= kSmallLMax) {
         // header: work-list counter, then the dense pass's tile ticket
         uint32_t *count = reinterpret_cast<uint32_t *>(ws);
@@ -24,7 +39,7 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
         if (e != cudaSuccess) return e;
         // 32-bit pass over the batch, then a 64-bit pass over the instances it listed
         return launch_small(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status,
-                            count, list, stream);
+                            count, list, pe, stream);
     }
     if (L <= kMidLMax) {
         // looped 32-bit pass (tile ticket + work list in the header), then the
@@ -35,8 +50,12 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
         uint32_t *tb = reinterpret_cast<uint32_t *>(ws + Workspace::table_offset(batch, L));
         cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(uint32_t), stream);
         if (e != cudaSuccess) return e;
+        e = mark(pe.start);
+        if (e != cudaSuccess) return e;
         e = launch_mid(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, ticket,
                        count, list, tb, stream);
+        if (e != cudaSuccess) return e;
+        e = mark(pe.stop);
         if (e != cudaSuccess) return e;
         if (L <= kSmemTableLMax) {  // tables of the listed instances in shared memory
             const int64_t grid = batch < 152 * 8 ? batch : 152 * 8;
@@ -56,9 +75,13 @@ cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *c
     uint32_t *tickets = busy + nslots;
     cudaError_t e = cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
     if (e != cudaSuccess) return e;
+    e = mark(pe.start);
+    if (e != cudaSuccess) return e;
     e = launch_deep(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, tickets,
                     busy, count, list, ws + Workspace::deep_slots_offset(batch, L), nslots,
                     stream);
+    if (e != cudaSuccess) return e;
+    e = mark(pe.stop);
     if (e != cudaSuccess) return e;
     return launch_group(forward, batch, L, comp, xfer, dt, makespan, bits, nseg, status, count,
                         list, ws + Workspace::group_tables_offset(batch, L),
@@ -189,6 +212,14 @@ const char *dc_status_string(dc_status s)
         case DC_ERR_INTERNAL: return "solver self-check failed";
     }
     return "unknown status";
+}
+
+dc_status dc_time_next_pass(cudaEvent_t start, cudaEvent_t stop)
+{
+    if ((start == nullptr) != (stop == nullptr)) return DC_ERR_NULL;
+    dc::t_pass_events.start = start;
+    dc::t_pass_events.stop = stop;
+    return DC_OK;
 }
 
 dc_status dc_roof_int_probe(int32_t variant, int32_t blocks, int32_t threads, int64_t iters,

@@ -74,6 +74,7 @@ _SIGNATURES = {
     "dc_greedy_backward_batch": (_I32, [_I64, _I32, _VP, _VP, _VP, _VP, _VP, _VP]),
     "dc_status_string": (ctypes.c_char_p, [_I32]),
     "dc_roof_int_probe": (_I32, [_I32, _I32, _I32, _I64, _VP, _VP]),
+    "dc_time_next_pass": (_I32, [_VP, _VP]),
 }
 
 
@@ -249,6 +250,16 @@ def dc_greedy_backward_batch(batch, L, bc, gt, dt, makespan, bits, stream=None) 
 def dc_roof_int_probe(variant, blocks, threads, iters, sink, stream=None) -> int:
     return int(lib().dc_roof_int_probe(int(variant), int(blocks), int(threads), int(iters),
                                        _ptr(sink), _stream(stream)))
+
+
+def dc_time_next_pass(start, stop) -> int:
+    """start, stop: torch.cuda.Event (recorded at least once, so that their CUDA
+    events exist), raw cudaEvent_t addresses, or None for both."""
+    def ev(e):
+        if e is None:
+            return None
+        return e if isinstance(e, int) else int(e.cuda_event)
+    return int(lib().dc_time_next_pass(ev(start), ev(stop)))
 
 
 # ------------------------------------------------------------ conveniences

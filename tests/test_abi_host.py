@@ -174,3 +174,11 @@ def test_generated_host_checks(lib):
     assert f(cfg, FAKE, None, None, None, FAKE, need) == dc.DC_ERR_NULL
     assert f(cfg, FAKE, FAKE, None, None, None, need) == dc.DC_ERR_WORKSPACE
     assert f(cfg, FAKE, FAKE, None, None, FAKE, need - 1) == dc.DC_ERR_WORKSPACE
+
+
+def test_time_next_pass_arguments(lib):
+    """The timing request takes both events or neither; the checks run on the
+    host (no event is touched until a schedule call uses the request)."""
+    assert dc.dc_time_next_pass(None, FAKE) == dc.DC_ERR_NULL
+    assert dc.dc_time_next_pass(FAKE, None) == dc.DC_ERR_NULL
+    assert dc.dc_time_next_pass(None, None) == dc.DC_OK  # withdraws nothing pending
