@@ -229,7 +229,7 @@ PassEvents take_pass_events();  // this thread's request, cleared (dynacomm_abi.
 cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *comp,
                             const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                             uint32_t *bits, int32_t *nseg, int32_t *status, void *workspace,
-                            cudaStream_t stream);
+                            const PassEvents &pe, cudaStream_t stream);
 cudaError_t launch_small(bool forward, int64_t batch, int L, const int64_t *comp,
                          const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                          uint32_t *bits, int32_t *nseg, int32_t *status,

@@ -25,10 +25,9 @@ PassEvents take_pass_events()
 cudaError_t launch_schedule(bool forward, int64_t batch, int L, const int64_t *comp,
                             const int64_t *xfer, const int64_t *dt, int64_t *makespan,
                             uint32_t *bits, int32_t *nseg, int32_t *status, void *workspace,
-                            cudaStream_t stream)
+                            const PassEvents &pe, cudaStream_t stream)
 {
     unsigned char *ws = static_cast<unsigned char *>(workspace);
-    const PassEvents pe = take_pass_events();
     // events around the first pass of a looped or deep-chain solve
     auto mark = [&](cudaEvent_t ev) { return ev ? cudaEventRecord(ev, stream) : cudaSuccess; };
     if (L <= kSmallLMax) {
@@ -95,13 +94,14 @@ dc_status schedule(bool forward, int64_t batch, int32_t L, const int64_t *comp,
                    int32_t *nseg, int32_t *status, void *workspace, size_t workspace_bytes,
                    cudaStream_t stream)
 {
+    const PassEvents pe = take_pass_events();  // used up by this call, whatever it returns
     if (batch < 0 || L < 1 || L > DC_L_MAX || batch > int64_t(0xffffffffll))
         return DC_ERR_BAD_SHAPE;
     if (batch == 0) return DC_OK;
     if (!comp || !xfer || !dt || !makespan || (!bits && words_for(L) > 0)) return DC_ERR_NULL;
     if (!workspace || workspace_bytes < Workspace::bytes(batch, L)) return DC_ERR_WORKSPACE;
     const cudaError_t e = launch_schedule(forward, batch, L, comp, xfer, dt, makespan, bits,
-                                          nseg, status, workspace, stream);
+                                          nseg, status, workspace, pe, stream);
     return e == cudaSuccess ? DC_OK : DC_ERR_CUDA;
 }
 

@@ -52,6 +52,7 @@ extern "C" dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_
                                               cudaStream_t stream)
 {
     const dc::NvtxRange nvtx("dc_schedule_batch_static");
+    const dc::PassEvents pe = dc::take_pass_events();  // a timing request is used up here too
     if ((dir != 0 && dir != 1) || batch < 0 || L < 1 || L > dc::kSmallLMax)
         return DC_ERR_BAD_SHAPE;
     if (batch > dc::kStaticMaxBatch) return DC_ERR_WORKSPACE;  // beyond the static scratch
@@ -61,6 +62,6 @@ extern "C" dc_status dc_schedule_batch_static(int32_t dir, int64_t batch, int32_
     void *scratch = nullptr;
     if (dc::static_scratch(&scratch) != cudaSuccess) return DC_ERR_CUDA;
     const cudaError_t e = dc::launch_schedule(dir == 0, batch, L, comp, xfer, dt, makespan,
-                                              bits, nseg, status, scratch, stream);
+                                              bits, nseg, status, scratch, pe, stream);
     return e == cudaSuccess ? DC_OK : DC_ERR_CUDA;
 }

@@ -56,3 +56,24 @@ def test_first_pass_events(dc, L, B):
     torch.cuda.synchronize()
     for k in ("makespan", "bits", "nseg", "status"):
         assert torch.equal(out[k], ref[k]), k
+
+
+def test_request_used_up_by_a_failing_call(dc):
+    """A schedule call that fails its host checks still uses up the request: the
+    next, valid call records nothing into the events."""
+    import torch
+    comp, xfer, dt = wl.random_instances(5, 300, 16)
+    c, x, d = (torch.from_numpy(a).cuda() for a in (comp, xfer, dt))
+    sch = dc.Scheduler(300, 16)
+    k0, k1, after = _events(torch, 3)
+    assert dc.dc_time_next_pass(k0, k1) == dc.DC_OK
+    o = sch.out[0]
+    bad = dc.dc_schedule_forward_batch(300, 16, c, x, d, o["makespan"], o["bits"], o["nseg"],
+                                       o["status"], sch.workspace, 0)  # workspace too short
+    assert bad == dc.DC_ERR_WORKSPACE
+    after.record()
+    torch.cuda.synchronize()
+    before = k1.elapsed_time(after)
+    sch.run(0, c, x, d)
+    torch.cuda.synchronize()
+    assert k1.elapsed_time(after) == pytest.approx(before)
