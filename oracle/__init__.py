@@ -22,7 +22,10 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "dynacomm_oracle.c")
 _SRC_GREEDY = os.path.join(_HERE, "greedy_oracle.c")
 _HDR = os.path.join(_HERE, "dynacomm_oracle.h")
-_LIB = os.path.join(_HERE, "liboracle.so")
+# DC_ORACLE_LIB names a library built from planted-mistake copies of these
+# sources; only tests/test_oracle_mutations.py sets it, in child processes
+_LIB_OVERRIDE = os.environ.get("DC_ORACLE_LIB")
+_LIB = _LIB_OVERRIDE or os.path.join(_HERE, "liboracle.so")
 
 LAYERS_FIXED, LAYERS_UNIFORM, LAYERS_LOGUNIFORM = 0, 1, 2
 DIST_UNIFORM, DIST_LOGUNIFORM = 0, 1
@@ -30,6 +33,8 @@ DIST_UNIFORM, DIST_LOGUNIFORM = 0, 1
 
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (plain C99, -O2, pthreads)."""
+    if _LIB_OVERRIDE:
+        return _LIB_OVERRIDE
     stale = force or not os.path.exists(_LIB) or any(
         os.path.getmtime(p) > os.path.getmtime(_LIB) for p in (_SRC, _SRC_GREEDY, _HDR))
     if stale:
