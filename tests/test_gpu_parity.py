@@ -79,6 +79,18 @@ def test_dp_random_parity(dc, L, kind):
         _check_direction(dc, d, comp, xfer, dt, f"L={L} {kind} dir={d}")
 
 
+@pytest.mark.parametrize("L", [9, 11, 12, 13, 14, 15, 16])
+def test_dp_many_tiles_per_warp(dc, L):
+    """Batches that give every resident warp of the short-L pass several tiles and
+    a ragged last one: the shared-area design (L < 12) and the split design with
+    its ticket and the next tile staged while one is solved (12 <= L <= 16; odd L
+    copies 8-byte words), against the oracle on every instance."""
+    B = 480_007
+    comp, xfer, dt = wl.random_instances(7000 + L, B, L)
+    for d in (FWD, BWD):
+        _check_direction(dc, d, comp, xfer, dt, f"L={L} B={B} dir={d}")
+
+
 @pytest.mark.parametrize("L", [257, 258, 300, 333, 512, 600])
 @pytest.mark.parametrize("kind", ["tie", "uni", "skew"])
 def test_dp_deep_random_parity(dc, L, kind):
