@@ -126,19 +126,38 @@ def load_json(path):
         return None
 
 
-def dp_source_hash() -> str:
-    """Hash of the code (comments and blank space removed) of the sources the
-    short-L dense pass is built from, which a traffic record must match to be
-    reported."""
+# the sources each first-pass kernel is built from, by the L it serves
+FIRST_PASS_SOURCES = {
+    "small_dense_kernel": ("dp_small.cu", "dp_small.cuh", "gen_device.cuh", "common.cuh"),
+    "mid_kernel": ("dp_mid.cu", "common.cuh"),
+    "deep_kernel": ("dp_deep.cu", "common.cuh"),
+}
+
+
+def dp_source_hash(kernel: str = "small_dense_kernel") -> str:
+    """Hash of the code (comments and blank space removed) of the sources a first
+    pass is built from, which a traffic record must match to be reported."""
     import hashlib
     import re
     h = hashlib.sha256()
-    for name in ("dp_small.cu", "dp_small.cuh", "gen_device.cuh", "common.cuh"):
+    for name in FIRST_PASS_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2101_07968_gb300", "csrc", name)) as f:
             code = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
         code = re.sub(r"//[^\n]*", "", code)
         h.update("".join(code.split()).encode())
     return h.hexdigest()[:16]
+
+
+def traffic_record(workload: str, L: int):
+    """DRAM bytes of one direction's first pass from profiles/dp_traffic.json, if
+    a record for this workload matches the kernel's current sources."""
+    data = load_json(TRAFFIC_PATH) or {}
+    kernel = first_pass_kernel(L)
+    for rec in data.get("records", []):
+        if (rec.get("workload") == workload and rec.get("kernel") == kernel
+                and rec.get("source_hash") == dp_source_hash(kernel)):
+            return rec.get("bytes_per_direction")
+    return None
 
 
 def first_pass_kernel(L: int) -> str:
@@ -667,10 +686,7 @@ def run_ours(args):
     # ALU roof from unit counts: 4 x 16 integer-ALU lanes per SM per clock, the
     # 32-bit passes spend 1.5 ALU instructions per transition
     peak = sms * 64 * MAX_SM_MHZ * 1e6 / ALU_OPS_PER_TRANSITION / 1e9
-    traffic = None
-    tr = load_json(TRAFFIC_PATH)
-    if tr and tr.get("workload") == args.workload and tr.get("source_hash") == dp_source_hash():
-        traffic = tr.get("bytes_per_launch")
+    traffic = traffic_record(args.workload, L)
     hbm_peak = (load_json(PEAKS_PATH) or {}).get("hbm_gbs", 6800.0)
     dp_gbs = dp_bytes(L) * (2 * B - listed[0] - listed[1]) / first_s / 1e9
     # kernels of this library per step: the generator; per direction the first
