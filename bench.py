@@ -786,19 +786,22 @@ def run_e2e(dc, torch, prof, sched, B, L, W, dev, args, barrier, world):
     for d in (0, 1):  # the pipelined results equal the device-resident path's
         if not torch.equal(host_out[(d, "makespan")], sched.out[d]["makespan"].cpu()):
             raise RuntimeError("host pipeline disagrees with the device path")
-    steps = max(1, min(args.steps, 5))
+    steps = max(1, min(args.steps, 10))
     barrier()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(steps):
+    # one event per step boundary on the caller's stream (each run ends by joining
+    # its streams into it), so that the spread of the steps is visible too
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    ev[0].record()
+    for s in range(steps):
         pipe.run(host_in, host_out)
-    t1.record()
+        ev[s + 1].record()
     torch.cuda.synchronize()
     barrier()
-    ms = max_over_ranks(t0.elapsed_time(t1) / steps, dev)
+    per_step = [ev[s].elapsed_time(ev[s + 1]) for s in range(steps)]
+    ms = max_over_ranks(ev[0].elapsed_time(ev[steps]) / steps, dev)
     return {"value": B * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps,
+            "ms_step_min_max": [min(per_step), max(per_step)],
             "path": f"pinned host profiles -> dynacomm.HostPipeline ({pipe.chunks} "
                     f"piece{'s' if pipe.chunks != 1 else ''}, "
                     "copies overlapped with dc_schedule_forward/backward_batch and "
