@@ -98,7 +98,7 @@ __global__ void __launch_bounds__(32, dense_min_ctas(L))
         if (st != DC_OK) {
             write_failure(st, i, W, makespan, bits, nseg, status);
         } else if (wide ||
-                   !solve_uv<L, FWD>(U, V, int32_t(dti), xraw, lw, i, makespan, bits, nseg, status)) {
+                   !solve_uv<L>(FWD, U, V, int32_t(dti), xraw, lw, i, makespan, bits, nseg, status)) {
             // 64-bit values, or a traceback deeper than the kept columns: work list
             const uint32_t at = atomicAdd(wide_count, 1u);
             if (DC_CHECK(int64_t(at) < batch)) wide_list[at] = uint32_t(i);

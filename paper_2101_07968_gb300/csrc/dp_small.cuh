@@ -253,18 +253,25 @@ __device__ __forceinline__ int32_t min_fold3(const int32_t (&c)[N], int cnt)
     return min(a, b);
 }
 
-template <int L, bool FWD>
-__device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
-                                       int32_t dt, int32_t fcL, int32_t *lw, int32_t &bestV,
-                                       int &best_s)
+// The direction `fwd` is an argument: the dense passes pass a compile-time
+// constant, which folds every choice below away; the fused pass solves both
+// directions with one copy of this code.
+template <int L>
+__device__ __forceinline__ void fill_e(const bool fwd, const int32_t (&U)[L + 1],
+                                       const int32_t (&V)[L + 1], int32_t dt, int32_t fcL,
+                                       int32_t *lw, int32_t &bestV, int &best_s)
 {
     using K = Tab32<L>;
     // forward: U = Q, V = G, col = A; backward: U = BC - dt, V = NGT, col = F
     const int32_t dt2 = 2 * dt;
+    const int32_t c1 = fwd ? fcL - dt : dt;  // column 1 is U + c1
+    const int32_t sdt = fwd ? -dt : dt;      // column n is its minimum + sdt
+    const int32_t uL = fwd ? U[L] : 0;       // row L's minimum less uL: B[L][n] or F[L][n] - dt
+    const int32_t step = fwd ? dt : 0, base = fwd ? 0 : dt2;
     int32_t col[L + 1];
 #pragma unroll
-    for (int m = 1; m <= L; ++m) col[m] = FWD ? fcL + U[m] - dt : U[m] + dt;
-    bestV = FWD ? fcL + dt : U[L] + dt2;
+    for (int m = 1; m <= L; ++m) col[m] = U[m] + c1;
+    bestV = fwd ? fcL + dt : U[L] + dt2;
     best_s = 1;
 #pragma unroll
     for (int n = 2; n <= L; ++n) {
@@ -277,11 +284,11 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
 #pragma unroll
             for (int j = 0; j < cnt; ++j) c[j] = __viaddmax_s32(u, V[n - 1 + j], col[n - 1 + j]);
             const int32_t b = min_fold3<L>(c, cnt);
-            if (m == L) last = FWD ? b - U[L] : b;
-            col[m] = FWD ? b - dt : b + dt;
+            if (m == L) last = b - uL;
+            col[m] = b + sdt;
             if (n <= K::kLast) lw[32 * (1 + cell2(L, m, n))] = col[m];
         }
-        const int32_t v = FWD ? last + n * dt : last + dt2;  // X[L][n] - P[L] or X[L][n] - S[L]
+        const int32_t v = last + n * step + base;  // X[L][n] - P[L] or X[L][n] - S[L]
         if (v < bestV) {  // strict: the lowest n wins ties
             bestV = v;
             best_s = n;
@@ -294,11 +301,11 @@ __device__ __forceinline__ void fill_e(const int32_t (&U)[L + 1], const int32_t 
 // prefix; backward: U = compute prefix - dt, V = -capped transfer prefix) and the raw
 // transfer sum. Returns false (writing nothing) when the traceback needs a column
 // the pass did not keep.
-template <int L, bool FWD>
-__device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_t (&V)[L + 1],
-                                         int32_t dt, uint64_t xraw, int32_t *lw, int64_t i,
-                                         int64_t *makespan, uint32_t *bits, int32_t *nseg,
-                                         int32_t *status)
+template <int L>
+__device__ __forceinline__ bool solve_uv(const bool fwd, const int32_t (&U)[L + 1],
+                                         const int32_t (&V)[L + 1], int32_t dt, uint64_t xraw,
+                                         int32_t *lw, int64_t i, int64_t *makespan,
+                                         uint32_t *bits, int32_t *nseg, int32_t *status)
 {
     using K = Tab32<L>;
     constexpr int W = (L - 1 + 31) / 32;
@@ -307,7 +314,7 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
     for (int m = 0; m <= L; ++m) lw[32 * (K::kOffU + m)] = U[m];  // the traceback reads U[m]
     int32_t bestV;
     int s;
-    fill_e<L, FWD>(U, V, dt, fcL, lw, bestV, s);
+    fill_e<L>(fwd, U, V, dt, fcL, lw, bestV, s);
     if (s - 1 > K::kLast && s - 1 >= 2) return false;
 
     // from (L, s) step to the lowest k whose candidate equals the cell, set
@@ -319,11 +326,11 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
     uint32_t word = 0;
     int err = 0;
     int m = L, n = s;
-    int32_t target = FWD ? bestV - s * dt + U[L] : bestV - 2 * dt;  // B[L][s] + Q[L] or F[L][s] - dt
+    int32_t target = fwd ? bestV - s * dt + U[L] : bestV - 2 * dt;  // B[L][s] + Q[L] or F[L][s] - dt
     // column 1 is U shifted by off1 (A[k][1] = FC[L] + U[k] - dt forward, F[k][1] =
     // U[k] + dt backward): its step reads U and compares the candidate and the
     // cell both less off1, max(u + V, f + off1) = max(u - off1 + V, f) + off1
-    const int32_t off1 = FWD ? fcL - dt : dt;
+    const int32_t off1 = fwd ? fcL - dt : dt;
     while (n > 1) {
         const int nm1 = n - 1;
         const int32_t off = nm1 == 1 ? off1 : 0;
@@ -344,7 +351,7 @@ __device__ __forceinline__ bool solve_uv(const int32_t (&U)[L + 1], const int32_
         const int k = __ffs(int(hit)) - 1;
         word |= 1u << ((k - 1) & 31);
         const int32_t fk = lds(lw, base + k) + off;  // the cell (k, n-1): B + Q[k] = A + dt, or F - dt
-        target = FWD ? fk + dt : fk - dt;
+        target = fwd ? fk + dt : fk - dt;
         m = k;
         n = nm1;
     }
