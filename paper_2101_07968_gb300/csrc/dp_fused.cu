@@ -3,10 +3,6 @@
 // profile generator's device functions instead of being read from memory.
 #include "dp_small.cuh"
 
-#ifndef DC_FUSED_PAIR
-#define DC_FUSED_PAIR 1
-#endif
-
 namespace dc {
 namespace {
 
@@ -20,7 +16,7 @@ namespace {
 // runs once per direction (two unrolled copies overflow the instruction cache).
 // Each direction has its own list pass, which regenerates the listed instances'
 // rows.
-// workspace: [0, 256) the two list counters and the two tile tickets,
+// workspace: [0, 256) the two list counters and the tile ticket,
 // [256, 256 + 8 batch) the two lists, then the generator's tables
 inline size_t fused_tables_offset(int64_t batch) { return (256 + 8 * size_t(batch) + 255) / 256 * 256; }
 
@@ -29,7 +25,7 @@ struct FusedOut {
     uint32_t *bits[2];
     int32_t *nseg[2], *status[2];
     uint32_t *wide_count[2], *wide_list[2];
-    uint32_t *ticket[2];  // tiles handed out per direction (zero before the launches)
+    uint32_t *ticket;  // tiles handed out (zero before the launch)
 };
 
 // The generator's lookup tables, copied once per call from the parameter block
@@ -49,86 +45,6 @@ __global__ void __launch_bounds__(256) copy_tables_kernel(const __grid_constant_
     for (int j = threadIdx.x; j < kFixedMax; j += blockDim.x) {
         t->l0[j] = g.layer0[j];
         t->l1[j] = g.layer1[j];
-    }
-}
-
-template <int L, bool FWD>
-__device__ __forceinline__ void fused_direction(const GenParams &g, const GenTables *t,
-                                                const InstanceDraws &d,
-                                                int64_t gi, int64_t i, bool active, int64_t *stC,
-                                                int64_t *stX, int32_t *lw, int lane,
-                                                const FusedOut &o)
-{
-    using K = Tab32<L>;
-    constexpr int W = (L - 1 + 31) / 32;
-    constexpr int dir = FWD ? 0 : 1;
-    __syncwarp();  // every lane is done with the area (the table of the other direction)
-    if (active) {
-        // rolled from kSplitMinL on: unrolled, the generator's divisions and the
-        // DP overflow the instruction cache (no_instruction leads the stalls)
-#pragma unroll (L >= kSplitMinL ? 1 : L)
-        for (int l = 0; l < L; ++l) {
-            int64_t params, flops, f, b, x;
-            layer_draws(g, t->l0, t->l1, gi, l, params, flops);
-            layer_costs(g, d, params, flops, f, b, x);
-            stC[lane * K::kStride + l] = FWD ? f : b;
-            stX[lane * K::kStride + l] = x;
-        }
-    }
-    const int64_t dti = active ? d.dt : 0;
-    int32_t U[L + 1], V[L + 1];
-    uint64_t xraw;
-    bool wide;
-    int st;
-    row_uv<L, FWD>(stC + lane * K::kStride, stX + lane * K::kStride, dti, U, V, xraw, wide, st);
-    __syncwarp();  // rows read: the lanes' table slices may be written
-    if (!active) return;
-    if (st != DC_OK) {
-        write_failure(st, i, W, o.makespan[dir], o.bits[dir], o.nseg[dir], o.status[dir]);
-    } else if (wide || !solve_uv<L>(FWD, U, V, int32_t(dti), xraw, lw, i, o.makespan[dir],
-                                         o.bits[dir], o.nseg[dir], o.status[dir])) {
-        const uint32_t at = atomicAdd(o.wide_count[dir], 1u);
-        if (DC_CHECK(int64_t(at) < g.batch)) o.wide_list[dir][at] = uint32_t(i);
-    }
-}
-
-template <int L, bool FWD>
-__global__ void __launch_bounds__(32, DC_SMALL_MINB)
-    fused_dense_kernel(const __grid_constant__ GenParams g, const GenTables *t, const FusedOut o)
-{
-    using K = Tab32<L>;
-    extern __shared__ __align__(16) unsigned char smem[];
-    const int lane = threadIdx.x;
-    int64_t *stC = reinterpret_cast<int64_t *>(smem);
-    int64_t *stX = stC + 32 * K::kStride;
-    int32_t *lw = reinterpret_cast<int32_t *>(smem) + lane;
-    const int64_t tiles = (g.batch + 31) / 32;
-    pdl_trigger();
-    auto solve_tile = [&](int64_t tile) {
-        const int64_t i = tile * 32 + lane;
-        const bool active = i < g.batch;
-        const int64_t gi = g.inst0 + i;
-        InstanceDraws d = {};
-        if (active) d = instance_draws(g, t->rate, t->bw, gi);
-        fused_direction<L, FWD>(g, t, d, gi, i, active, stC, stX, lw, lane, o);
-    };
-    if constexpr (L >= kSplitMinL) {
-        // tiles from a ticket, the next claimed while this one is solved (as in
-        // the dense pass: warps sharing a sub-partition progress at different rates)
-        uint32_t *ticket = o.ticket[FWD ? 0 : 1];
-        auto claim = [&]() {
-            uint32_t v = 0;
-            if (lane == 0) v = atomicAdd(ticket, 1u);
-            return v;
-        };
-        int64_t tile = int64_t(__shfl_sync(0xffffffffu, claim(), 0));
-        while (tile < tiles) {
-            const uint32_t next_raw = claim();
-            solve_tile(tile);
-            tile = int64_t(__shfl_sync(0xffffffffu, next_raw, 0));
-        }
-    } else {
-        for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) solve_tile(tile);
     }
 }
 
@@ -226,7 +142,7 @@ __global__ void __launch_bounds__(32, DC_SMALL_MINB)
         // tiles from a ticket, the next claimed while this one is solved
         auto claim = [&]() {
             uint32_t v = 0;
-            if (lane == 0) v = atomicAdd(o.ticket[0], 1u);
+            if (lane == 0) v = atomicAdd(o.ticket, 1u);
             return v;
         };
         int64_t tile = int64_t(__shfl_sync(0xffffffffu, claim(), 0));
@@ -300,39 +216,10 @@ cudaError_t launch_fused_list(const GenParams &g, const GenTables *t, const Fuse
     return cudaLaunchKernelEx(&lc, fused_list_kernel<L, FWD>, g, t, o);
 }
 
-template <int L, bool FWD>
-cudaError_t launch_fused_dir(const GenParams &g, const GenTables *t, const FusedOut &o,
-                             cudaStream_t stream)
-{
-    static DeviceCache resident;  // single-warp CTAs of the fused kernel per SM
-    int per_sm = 0;
-    cudaError_t le = resident.get(per_sm, [](int &n) {
-        cudaError_t e = cudaFuncSetAttribute(fused_dense_kernel<L, FWD>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             Tab32<L>::kSharedBytes);
-        if (e != cudaSuccess) return e;
-        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fused_dense_kernel<L, FWD>, 32,
-                                                             Tab32<L>::kSharedBytes);
-    });
-    if (le != cudaSuccess) return le;
-    const int64_t tiles = (g.batch + 31) / 32;
-    int64_t grid = int64_t(sm_count()) * per_sm;
-    if (grid > tiles) grid = tiles;
-    fused_dense_kernel<L, FWD><<<unsigned(grid), 32, Tab32<L>::kSharedBytes, stream>>>(g, t, o);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    return launch_fused_list<L, FWD>(g, t, o, stream);
-}
-
 template <int L>
 cudaError_t launch_fused_L(const GenParams &g, const GenTables *t, const FusedOut &o,
                            cudaStream_t stream)
 {
-    if (!DC_FUSED_PAIR) {
-        cudaError_t e = launch_fused_dir<L, true>(g, t, o, stream);
-        if (e != cudaSuccess) return e;
-        return launch_fused_dir<L, false>(g, t, o, stream);
-    }
     static DeviceCache resident;  // single-warp CTAs of the pair kernel per SM
     int per_sm = 0;
     cudaError_t le = resident.get(per_sm, [](int &n) {
@@ -374,9 +261,9 @@ cudaError_t launch_fused(const GenParams &g, int64_t *makespan, uint32_t *bits, 
         o.status[d] = status ? status + d * B : nullptr;
         o.wide_count[d] = reinterpret_cast<uint32_t *>(ws) + d;
         o.wide_list[d] = reinterpret_cast<uint32_t *>(ws + 256) + d * B;
-        o.ticket[d] = reinterpret_cast<uint32_t *>(ws) + 2 + d;
     }
-    cudaError_t e = cudaMemsetAsync(ws, 0, 4 * sizeof(uint32_t), stream);
+    o.ticket = reinterpret_cast<uint32_t *>(ws) + 2;
+    cudaError_t e = cudaMemsetAsync(ws, 0, 3 * sizeof(uint32_t), stream);
     if (e != cudaSuccess) return e;
     GenTables *t = reinterpret_cast<GenTables *>(ws + fused_tables_offset(B));
     copy_tables_kernel<<<1, 256, 0, stream>>>(g, t);
