@@ -38,6 +38,11 @@ def _configs():
     big = wl.with_batch(tiny, 20_011, inst0=777)
     big.update(dt_lo=10 ** 9, dt_hi=10 ** 12)  # bounds above 2^31: the list pass
     out.append(("huge_dt", big))
+    # bounds on both sides of 2^31 - 1: 32-bit and listed instances side by side,
+    # and a few listed in the backward direction only (its compute is larger)
+    mixed = wl.with_batch(tiny, 20_011, inst0=555)
+    mixed.update(dt_lo=2 * 10 ** 8, dt_hi=4 * 10 ** 8)
+    out.append(("mixed_dt", mixed))
     return out
 
 
@@ -67,6 +72,15 @@ def test_fused_equals_unfused(dc, name, cfg):
             assert np.array_equal(fused["bits"][d][:n, :W].cpu().numpy().view(np.uint32), exp["bits"])
     if name == "huge_dt":  # the list pass ran: some bound exceeds 2^31
         assert int((L * po["dt"] + po["fc"].sum(1)).max()) > 2 ** 31
+    if name == "mixed_dt":  # the batch holds all three kinds of instance
+        f = {k: prof[k].cpu().numpy() for k in ("fc", "pt", "bc", "gt", "dt")}
+
+        def wide(c, x):  # the capped bound of the shifted 32-bit form
+            tc = f[c].sum(1)
+            return L * f["dt"] + tc + np.minimum(f[x], tc[:, None]).sum(1) > 2 ** 31 - 1
+
+        wf, wb = wide("fc", "pt"), wide("bc", "gt")
+        assert (~wf & ~wb).any() and (wf & wb).any() and (wb & ~wf).any()
 
 
 def test_fused_errors(dc):
