@@ -2,7 +2,10 @@
 dc_profile_gen, then dc_schedule_forward_batch and dc_schedule_backward_batch on
 the profiles it wrote. Every output bit-exact; a sample also against the oracle
 directly. Configurations cover the fixed CNN shapes, per-instance layer draws,
-short L, and latencies large enough that instances take the 64-bit list pass.
+short L, latencies large enough that every instance takes the 64-bit list pass,
+batches that mix 32-bit and listed instances (some listed in one direction
+only, through large latencies or large compute), and optima deeper than the
+kept traceback columns.
 """
 import os
 
@@ -43,6 +46,15 @@ def _configs():
     mixed = wl.with_batch(tiny, 20_011, inst0=555)
     mixed.update(dt_lo=2 * 10 ** 8, dt_hi=4 * 10 ** 8)
     out.append(("mixed_dt", mixed))
+    # the same through large compute at ordinary latencies: optima of 2-5 segments
+    # on both sides of the bound, compute costs above 2^31 / L (the 64-bit prefix)
+    heavy = wl.with_batch(tiny, 20_011, inst0=999)
+    heavy.update(flops_lo=10 ** 9, flops_hi=10 ** 12, rate_lo=10 ** 3, rate_hi=10 ** 4)
+    out.append(("mixed_wide", heavy))
+    # optima of up to 8 segments: those deeper than the kept columns are listed
+    deep = wl.with_batch(tiny, 20_011, inst0=333)
+    deep.update(flops_lo=10 ** 9, flops_hi=10 ** 11, rate_lo=10 ** 3, rate_hi=10 ** 4)
+    out.append(("deep_s", deep))
     return out
 
 
@@ -70,9 +82,11 @@ def test_fused_equals_unfused(dc, name, cfg):
         assert np.array_equal(fused["nseg"][d][:n].cpu().numpy(), exp["nseg"])
         if W:
             assert np.array_equal(fused["bits"][d][:n, :W].cpu().numpy().view(np.uint32), exp["bits"])
+        if name == "deep_s":  # some tracebacks need more than the kept columns 1..4
+            assert int(exp["nseg"].max()) > 5
     if name == "huge_dt":  # the list pass ran: some bound exceeds 2^31
         assert int((L * po["dt"] + po["fc"].sum(1)).max()) > 2 ** 31
-    if name == "mixed_dt":  # the batch holds all three kinds of instance
+    if name in ("mixed_dt", "mixed_wide"):  # the batch holds all three kinds of instance
         f = {k: prof[k].cpu().numpy() for k in ("fc", "pt", "bc", "gt", "dt")}
 
         def wide(c, x):  # the capped bound of the shifted 32-bit form
