@@ -721,6 +721,9 @@ def run_ours(args):
                             kernel_ms={"forward": fwd_k_ms, "backward": bwd_k_ms},
                             listed_to_work_list={"forward": listed[0], "backward": listed[1]},
                             traffic=traffic, dp_call=dp_call)
+    if traffic is None:
+        roofline["traffic_note"] = ("no DRAM record in profiles/dp_traffic.json matches this "
+                                    "workload and the current sources of its first-pass kernel")
     clocks = clk.summary() if rank == 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
